@@ -1,0 +1,246 @@
+/*
+ * refadapt.h — C ABI of the RefAdapt-DiT hot path on one GB300 (sm_103a).
+ *
+ * RefAdapt-DiT (training-free reference reuse for reference-conditioned
+ * diffusion transformers): every DiT block runs joint attention over
+ * [text; reference; target] tokens. A block that reuses skips the reference
+ * query rows and lets text and target queries attend to reference K/V cached
+ * at the block's last materialisation; the first block whose head-mean score
+ * D x M reaches theta reactivates and every deeper block recomputes
+ * (paper Sec. 4, Algorithm 1).
+ *
+ * Conventions for every entry point:
+ *  - All device pointers are caller-owned; the library allocates no device
+ *    memory. Every call is asynchronous on `stream` (a cudaStream_t passed as
+ *    void*; NULL = the legacy default stream) and performs no host sync.
+ *  - Invalid arguments return RA_EINVAL before anything is launched;
+ *    refadapt_last_error() then holds a one-line reason (thread-local).
+ *  - A failed launch returns RA_ECUDA. A device-side wait that exceeded its
+ *    time budget sets bit 0 of the caller's error word (see
+ *    refadapt_check_error), never traps, and leaves the context usable.
+ *  - No exceptions cross the ABI; nothing calls exit().
+ *  - bf16 tensors are described by ra_seg: element (b, h, n, c) lives at
+ *    ptr + b*stride_b + h*stride_h + n*stride_n + c (strides in elements,
+ *    c contiguous). ptr and every stride must be 16-byte aligned
+ *    (strides multiples of 8 elements).
+ */
+#ifndef REFADAPT_H
+#define REFADAPT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  RA_OK = 0,
+  RA_EINVAL = 1,        /* bad argument; nothing launched */
+  RA_EUNSUPPORTED = 2,  /* valid but not supported here (e.g. no sm_103 device) */
+  RA_ECUDA = 3,         /* a CUDA call failed */
+  RA_ETIMEOUT = 4       /* a device-side wait ran out of its budget */
+} ra_status;
+
+/* Block execution modes (paper Sec. 4 "Execution and cache state";
+ * Algorithm 1). REUSE: reference query rows skipped, text and target rows
+ * attend to cached reference K/V. BOUNDARY: the first crossing block; every
+ * row runs, reference K/V still from the cache, the cache is not updated.
+ * COMPUTE: a block deeper than the boundary; fresh reference K/V are written
+ * to the cache (a_b = t) and every row runs. FULL: bounded-age or step-0 full
+ * refresh; same work as COMPUTE. */
+typedef enum {
+  RA_MODE_REUSE = 0,
+  RA_MODE_BOUNDARY = 1,
+  RA_MODE_COMPUTE = 2,
+  RA_MODE_FULL = 3
+} ra_mode;
+
+/* Token roles (paper Sec. 3 "Setting"): R = reference rows, Y = the
+ * remaining active-generation rows, split here into text and target. */
+enum { RA_TEXT = 0, RA_REF = 1, RA_TGT = 2 };
+
+/* Rows of one Q tile of the attention kernel; mass partials come per tile. */
+#define RA_MASS_TILE_ROWS 128
+
+typedef struct {
+  void* ptr;          /* device, bf16 */
+  int64_t stride_b;   /* elements */
+  int64_t stride_h;   /* elements */
+  int64_t stride_n;   /* elements */
+  int32_t n;          /* rows (tokens) in this segment, >= 0 */
+  int32_t reserved;   /* set to 0 */
+} ra_seg;
+
+/* ------------------------------------------------------------------ attention
+ * refadapt_joint_attn — joint attention of one DiT block with the reference
+ * mass as a by-product.
+ *
+ * Computes, per sample b and head h, O = Softmax(scale * Q K^T + bias) V
+ * (paper Sec. 3.3, Attn(Q,K,V) = Softmax(QK^T / sqrt(d_h)) V) over the keys
+ * [text; ref; target], bidirectional, no mask. Query rows: text and target
+ * when mode[b] == RA_MODE_REUSE (reference rows skipped, their O rows left
+ * untouched; App. A.4 removes the two reference-query score regions), every
+ * row otherwise. The reference K/V segments are whatever the caller points
+ * k[RA_REF] / v[RA_REF] at — normally the block's cache slot, so reuse costs
+ * no copy.
+ *
+ * Mass (paper Eq. 4): for every executed query row q in the mass row set,
+ * the softmax probability summed over reference keys, l_ref(q) / l(q), is
+ * accumulated per 128-row Q tile into mass_partial[b][h][i] (fp32), i over
+ * the text tiles (ceil(n_text/128)) then the target tiles
+ * (ceil(n_tgt/128)); refadapt_mass_partial_len() gives the length. Mass row
+ * set: target rows (mass_rows = 0), or text + target rows (mass_rows = 1);
+ * partials of tiles outside the set are written as 0. M_{t,b,h} is the sum of
+ * a (b, h) row of partials divided by the number of mass rows (the gate does
+ * this). Every partial is written on every call, in a fixed reduction order
+ * (deterministic).
+ *
+ * Arguments:
+ *  q, k, v, o [3]   segments per role (RA_TEXT, RA_REF, RA_TGT). For each
+ *                   role all four must have the same n; n_tgt >= 1.
+ *                   q[RA_REF] / o[RA_REF] may have ptr NULL only if n_ref == 0
+ *                   or every sample reuses.
+ *  B, H, d          batch, heads, head dim; d in {64, 128}.
+ *  softmax_scale    > 0; pass 0 for 1/sqrt(d).
+ *  ref_logit_bias   device [H] fp32 or NULL: added to the logits of target
+ *                   query rows against reference keys (natural-log units).
+ *  mode             device [B] int32 (ra_mode) or NULL (= every row runs).
+ *  mass_partial     device [B][H][refadapt_mass_partial_len(n_text, n_tgt)].
+ *  err_word         device int32 or NULL; bit 0 set on a device timeout.
+ */
+typedef struct {
+  int32_t B, H, d;
+  int32_t mass_rows;
+  ra_seg q[3], k[3], v[3], o[3];
+  float softmax_scale;
+  int32_t reserved;
+  const float* ref_logit_bias;
+  const int32_t* mode;
+  float* mass_partial;
+  int32_t* err_word;
+} ra_attn_args;
+
+ra_status refadapt_joint_attn(const ra_attn_args* args, void* stream);
+
+int32_t refadapt_mass_partial_len(int32_t n_text, int32_t n_tgt);
+
+/* ------------------------------------------------------------------ Q change
+ * refadapt_q_delta — consecutive relative drift of the post-RoPE target
+ * query, per sample and head (paper Eq. 1 applied to Q^{Y,h}, Sec. 4
+ * "Runtime cues"):
+ *   D[b][h] = ||q_cur - q_prev||_F / (||q_prev||_F + eps)
+ * over the segment's n rows x d columns. Bandwidth-bound: reads both tensors
+ * once with 16-byte loads, fp32 per-thread sums, fp64 across threads and
+ * blocks in a fixed order (deterministic).
+ *
+ *  q_cur, q_prev    segments with equal n (>= 1); d in {64, 128}.
+ *  d_out            device [B][H] fp32.
+ *  workspace        device scratch of refadapt_q_delta_workspace_size(B, H)
+ *                   bytes, 16-byte aligned, zero-filled once before its first
+ *                   use; every call leaves it ready for the next. Calls that
+ *                   share a workspace must be stream-ordered.
+ */
+size_t refadapt_q_delta_workspace_size(int32_t B, int32_t H);
+ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
+                           float eps, float* d_out, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ------------------------------------------------------------------ gate
+ * Controller state of Algorithm 1 for one trajectory (opaque, device
+ * resident): a_full (step of the last full refresh), whether the current
+ * step is a full refresh, and per sample the reactivated latch and boundary.
+ */
+typedef struct ra_state ra_state;
+size_t refadapt_state_size(int32_t B);
+ra_status refadapt_state_init(ra_state* state, int32_t B, void* stream);
+
+/* refadapt_gate — one block's decision (paper Eqs. 12-13, App. A.2 head
+ * mean, bounded-age refresh of Sec. 4 / Algorithm 1), on the device.
+ *
+ * Must be called for blocks 0, 1, ... in order within a step. At b == 0 it
+ * opens step t: t == 0 forces FULL (and a_full = 0); else t - a_full >=
+ * delta_max forces FULL for every block of the step (and a_full = t); else
+ * the reactivated latch is cleared. Per sample: g_h = D[b][h] * M_{t-1,b,h}
+ * (M from the previous step's mass partials of this block), gbar = mean_h
+ * g_h; FULL if the step is a full refresh, COMPUTE if already reactivated,
+ * else BOUNDARY (and latch) if gbar >= theta — or b >= forced_boundary when
+ * forced_boundary >= 0 — else REUSE.
+ *
+ *  q_delta            device [B][H] (refadapt_q_delta for this step/block);
+ *                     may be NULL at t == 0.
+ *  mass_partial_prev  device [B][H][mass_partial_len] from step t-1, block b;
+ *                     may be NULL at t == 0.
+ *  mass_row_count     number of rows the partials cover (n_tgt, or
+ *                     n_text + n_tgt when mass_rows = 1).
+ *  mode_out           device [B] int32, read by refadapt_joint_attn and
+ *                     refadapt_ref_cache_update.
+ *  gbar_out, m_out    device [B] and [B][H] fp32 or NULL (logging; gbar is
+ *                     NaN at t == 0).
+ */
+typedef struct {
+  double theta;
+  int32_t t, b, B, H;
+  int32_t delta_max;
+  int32_t forced_boundary;
+  int32_t mass_partial_len;
+  int32_t mass_row_count;
+  const float* q_delta;
+  const float* mass_partial_prev;
+  ra_state* state;
+  int32_t* mode_out;
+  float* gbar_out;
+  float* m_out;
+} ra_gate_args;
+
+ra_status refadapt_gate(const ra_gate_args* args, void* stream);
+
+/* ------------------------------------------------------------------ cache
+ * refadapt_ref_cache_update — materialise a block's reference K/V into its
+ * cache slot (paper Eq. 11, Z_b = (H_b, K_b, V_b, a_b); Algorithm 1: a
+ * COMPUTE or FULL block updates K_b, V_b and sets a_b = t).
+ *
+ * For each sample b with mode[b] in {COMPUTE, FULL}: copies k_src -> k_cache,
+ * v_src -> v_cache and, when x_src is not NULL, x_src -> x_cache (the
+ * block's cached reference hidden state, any bf16 [B, x_heads, n, x_width]
+ * tensor), then sets a_b[b] = t. Samples in other modes are untouched. A copy
+ * whose source and destination pointers are equal is skipped (in-place
+ * producer). 16-byte vector copies.
+ *
+ *  k_*, v_*      segments [B, H, n_ref, d]; all n equal; d in {64, 128}.
+ *  x_src/x_cache optional segments [B, x_heads, n_ref, x_width];
+ *                x_width a multiple of 8.
+ *  mode          device [B] int32.
+ *  a_b           device [B] int32 or NULL.
+ */
+ra_status refadapt_ref_cache_update(const ra_seg* k_src, const ra_seg* v_src, const ra_seg* k_cache,
+                                    const ra_seg* v_cache, int32_t B, int32_t H, int32_t d,
+                                    const ra_seg* x_src, const ra_seg* x_cache, int32_t x_heads,
+                                    int32_t x_width, const int32_t* mode, int32_t t, int32_t* a_b,
+                                    void* stream);
+
+/* ------------------------------------------------------------------ misc */
+const char* refadapt_status_string(ra_status s);
+const char* refadapt_last_error(void);
+
+/* Budget, in nanoseconds, of every device-side mbarrier wait of kernels
+ * launched afterwards by this process (default 2e9). */
+void refadapt_set_wait_budget_ns(uint64_t ns);
+
+/* Synchronises `stream`, reads the device error word, clears it and returns
+ * RA_ETIMEOUT if a device wait ran out, RA_ECUDA on a CUDA error, else RA_OK. */
+ra_status refadapt_check_error(int32_t* err_word, void* stream);
+
+int32_t refadapt_version(void);
+
+/* Diagnostic for the timeout path: launches one thread that waits, with the
+ * given budget, on an mbarrier that nothing ever arrives at — the same bounded
+ * wait every kernel uses. The wait gives up, sets bit 0 of *err_word and the
+ * kernel returns normally, so refadapt_check_error then reports RA_ETIMEOUT
+ * with the context still usable. budget_ns is capped at 1e9. */
+ra_status refadapt_selftest_wait_timeout(int32_t* err_word, uint64_t budget_ns, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* REFADAPT_H */

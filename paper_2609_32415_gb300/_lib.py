@@ -1,0 +1,110 @@
+"""ctypes view of librefadapt.so: structures and prototypes of include/refadapt.h.
+
+The library is built in-tree by ``paper_2609_32415_gb300.build``. Loading fails
+loudly when it is missing: there is no CPU fallback for any entry point.
+"""
+import ctypes
+import os
+from ctypes import POINTER, c_double, c_float, c_int32, c_int64, c_size_t, c_uint64, c_void_p
+
+PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(PKG, "librefadapt.so")
+
+RA_OK, RA_EINVAL, RA_EUNSUPPORTED, RA_ECUDA, RA_ETIMEOUT = 0, 1, 2, 3, 4
+RA_MODE_REUSE, RA_MODE_BOUNDARY, RA_MODE_COMPUTE, RA_MODE_FULL = 0, 1, 2, 3
+RA_TEXT, RA_REF, RA_TGT = 0, 1, 2
+RA_MASS_TILE_ROWS = 128
+
+EXPORTED = (
+    "refadapt_joint_attn", "refadapt_mass_partial_len", "refadapt_q_delta_workspace_size",
+    "refadapt_q_delta", "refadapt_state_size", "refadapt_state_init", "refadapt_gate",
+    "refadapt_ref_cache_update", "refadapt_status_string", "refadapt_last_error",
+    "refadapt_set_wait_budget_ns", "refadapt_check_error", "refadapt_version",
+    "refadapt_selftest_wait_timeout",
+)
+
+
+class RaSeg(ctypes.Structure):
+    _fields_ = [("ptr", c_void_p), ("stride_b", c_int64), ("stride_h", c_int64),
+                ("stride_n", c_int64), ("n", c_int32), ("reserved", c_int32)]
+
+
+class RaAttnArgs(ctypes.Structure):
+    _fields_ = [("B", c_int32), ("H", c_int32), ("d", c_int32), ("mass_rows", c_int32),
+                ("q", RaSeg * 3), ("k", RaSeg * 3), ("v", RaSeg * 3), ("o", RaSeg * 3),
+                ("softmax_scale", c_float), ("reserved", c_int32),
+                ("ref_logit_bias", c_void_p), ("mode", c_void_p), ("mass_partial", c_void_p),
+                ("err_word", c_void_p)]
+
+
+class RaGateArgs(ctypes.Structure):
+    _fields_ = [("theta", c_double), ("t", c_int32), ("b", c_int32), ("B", c_int32), ("H", c_int32),
+                ("delta_max", c_int32), ("forced_boundary", c_int32), ("mass_partial_len", c_int32),
+                ("mass_row_count", c_int32), ("q_delta", c_void_p), ("mass_partial_prev", c_void_p),
+                ("state", c_void_p), ("mode_out", c_void_p), ("gbar_out", c_void_p),
+                ("m_out", c_void_p)]
+
+
+class RefAdaptError(RuntimeError):
+    def __init__(self, fn, status, msg):
+        super().__init__("%s failed: %s (%s)" % (fn, _status_name(status), msg))
+        self.status = status
+
+
+def _status_name(s):
+    return {0: "RA_OK", 1: "RA_EINVAL", 2: "RA_EUNSUPPORTED", 3: "RA_ECUDA", 4: "RA_ETIMEOUT"}.get(s, str(s))
+
+
+_lib = None
+
+
+def load():
+    """Load librefadapt.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(LIB_PATH):
+        raise RuntimeError(
+            "librefadapt.so is missing (%s): build it with `python -c \"import __graft_entry__ as g; "
+            "g.build()\"` or `python -m paper_2609_32415_gb300.build`; there is no CPU fallback" % LIB_PATH)
+    lib = ctypes.CDLL(LIB_PATH)
+    lib.refadapt_joint_attn.restype = c_int32
+    lib.refadapt_joint_attn.argtypes = [POINTER(RaAttnArgs), c_void_p]
+    lib.refadapt_mass_partial_len.restype = c_int32
+    lib.refadapt_mass_partial_len.argtypes = [c_int32, c_int32]
+    lib.refadapt_q_delta_workspace_size.restype = c_size_t
+    lib.refadapt_q_delta_workspace_size.argtypes = [c_int32, c_int32]
+    lib.refadapt_q_delta.restype = c_int32
+    lib.refadapt_q_delta.argtypes = [POINTER(RaSeg), POINTER(RaSeg), c_int32, c_int32, c_int32, c_float,
+                                     c_void_p, c_void_p, c_size_t, c_void_p]
+    lib.refadapt_state_size.restype = c_size_t
+    lib.refadapt_state_size.argtypes = [c_int32]
+    lib.refadapt_state_init.restype = c_int32
+    lib.refadapt_state_init.argtypes = [c_void_p, c_int32, c_void_p]
+    lib.refadapt_gate.restype = c_int32
+    lib.refadapt_gate.argtypes = [POINTER(RaGateArgs), c_void_p]
+    lib.refadapt_ref_cache_update.restype = c_int32
+    lib.refadapt_ref_cache_update.argtypes = [POINTER(RaSeg), POINTER(RaSeg), POINTER(RaSeg), POINTER(RaSeg),
+                                              c_int32, c_int32, c_int32, POINTER(RaSeg), POINTER(RaSeg),
+                                              c_int32, c_int32, c_void_p, c_int32, c_void_p, c_void_p]
+    lib.refadapt_status_string.restype = ctypes.c_char_p
+    lib.refadapt_status_string.argtypes = [c_int32]
+    lib.refadapt_last_error.restype = ctypes.c_char_p
+    lib.refadapt_last_error.argtypes = []
+    lib.refadapt_set_wait_budget_ns.restype = None
+    lib.refadapt_set_wait_budget_ns.argtypes = [c_uint64]
+    lib.refadapt_check_error.restype = c_int32
+    lib.refadapt_check_error.argtypes = [c_void_p, c_void_p]
+    lib.refadapt_version.restype = c_int32
+    lib.refadapt_version.argtypes = []
+    lib.refadapt_selftest_wait_timeout.restype = c_int32
+    lib.refadapt_selftest_wait_timeout.argtypes = [c_void_p, c_uint64, c_void_p]
+    _lib = lib
+    return lib
+
+
+def check(fn, status):
+    if status != RA_OK:
+        msg = load().refadapt_last_error().decode(errors="replace")
+        raise RefAdaptError(fn, status, msg)
+    return status

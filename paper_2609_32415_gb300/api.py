@@ -1,0 +1,155 @@
+"""Thin Python binding of the C ABI (include/refadapt.h), same names.
+
+Only argument marshalling happens here: torch tensors supply device memory and
+streams; every step of the computation runs in librefadapt.so's kernels.
+Tensors are [B, H, n, d] bf16 CUDA views with a contiguous last axis (any
+other strides, 16-byte aligned).
+"""
+import ctypes
+
+import torch
+
+from . import _lib
+from ._lib import RaAttnArgs, RaGateArgs, RaSeg, check
+
+__all__ = ["seg", "refadapt_joint_attn", "refadapt_mass_partial_len", "refadapt_q_delta",
+           "refadapt_q_delta_workspace_size", "refadapt_state_size", "refadapt_state_init",
+           "refadapt_gate", "refadapt_ref_cache_update", "refadapt_set_wait_budget_ns",
+           "refadapt_check_error", "refadapt_version", "refadapt_selftest_wait_timeout", "q_delta_workspace", "new_state",
+           "alloc_mass_partial"]
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    if isinstance(stream, torch.cuda.Stream):
+        return ctypes.c_void_p(stream.cuda_stream)
+    return ctypes.c_void_p(int(stream))
+
+
+def seg(t, n=None) -> RaSeg:
+    """ra_seg of a [B, H, n, d] bf16 CUDA tensor (None -> empty/absent segment)."""
+    if t is None:
+        return RaSeg(None, 0, 0, 0, int(n or 0), 0)
+    if t.dim() != 4 or t.dtype != torch.bfloat16 or not t.is_cuda or (t.shape[3] > 1 and t.stride(3) != 1):
+        raise ValueError("expected a [B, H, n, d] bf16 CUDA tensor with contiguous last axis, got %s %s %s"
+                         % (tuple(t.shape), t.dtype, t.device))
+    ptr = t.data_ptr() if t.numel() > 0 else 0
+    return RaSeg(ptr or None, t.stride(0), t.stride(1), t.stride(2), t.shape[2], 0)
+
+
+def refadapt_mass_partial_len(n_text, n_tgt) -> int:
+    return int(_lib.load().refadapt_mass_partial_len(int(n_text), int(n_tgt)))
+
+
+def alloc_mass_partial(B, H, n_text, n_tgt, device="cuda"):
+    return torch.zeros((B, H, refadapt_mass_partial_len(n_text, n_tgt)), dtype=torch.float32, device=device)
+
+
+def refadapt_joint_attn(q, k, v, o, mass_partial, mode=None, softmax_scale=0.0, ref_logit_bias=None,
+                        mass_rows=0, err_word=None, stream=None):
+    """q, k, v, o: sequences (text, ref, tgt) of [B, H, n, d] tensors; q[1] / o[1] may be None."""
+    lib = _lib.load()
+    B, H, _, d = k[2].shape
+    a = RaAttnArgs()
+    a.B, a.H, a.d, a.mass_rows = B, H, d, int(mass_rows)
+    for r in range(3):
+        n_r = k[r].shape[2]
+        a.q[r] = seg(q[r], n_r)
+        a.k[r] = seg(k[r])
+        a.v[r] = seg(v[r])
+        a.o[r] = seg(o[r], n_r)
+    a.softmax_scale = float(softmax_scale)
+    a.ref_logit_bias = _ptr(ref_logit_bias)
+    a.mode = _ptr(mode)
+    a.mass_partial = _ptr(mass_partial)
+    a.err_word = _ptr(err_word)
+    return check("refadapt_joint_attn", lib.refadapt_joint_attn(ctypes.byref(a), _stream(stream)))
+
+
+def refadapt_q_delta_workspace_size(B, H) -> int:
+    return int(_lib.load().refadapt_q_delta_workspace_size(int(B), int(H)))
+
+
+def q_delta_workspace(B, H, device="cuda"):
+    """A zero-filled workspace for refadapt_q_delta (reusable across calls)."""
+    return torch.zeros(refadapt_q_delta_workspace_size(B, H), dtype=torch.uint8, device=device)
+
+
+def refadapt_q_delta(q_cur, q_prev, d_out, workspace, eps=1e-6, stream=None):
+    lib = _lib.load()
+    B, H, _, d = q_cur.shape
+    sc, sp = seg(q_cur), seg(q_prev)
+    return check("refadapt_q_delta", lib.refadapt_q_delta(
+        ctypes.byref(sc), ctypes.byref(sp), B, H, d, float(eps), _ptr(d_out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def refadapt_state_size(B) -> int:
+    return int(_lib.load().refadapt_state_size(int(B)))
+
+
+def refadapt_state_init(state, B, stream=None):
+    return check("refadapt_state_init", _lib.load().refadapt_state_init(_ptr(state), int(B), _stream(stream)))
+
+
+def new_state(B, device="cuda", stream=None):
+    st = torch.empty(refadapt_state_size(B), dtype=torch.uint8, device=device)
+    refadapt_state_init(st, B, stream)
+    return st
+
+
+def refadapt_gate(t, b, state, mode_out, theta, delta_max, B, H, q_delta=None, mass_partial_prev=None,
+                  mass_row_count=0, forced_boundary=-1, gbar_out=None, m_out=None, stream=None):
+    a = RaGateArgs()
+    a.theta = float(theta)
+    a.t, a.b, a.B, a.H = int(t), int(b), int(B), int(H)
+    a.delta_max = int(delta_max)
+    a.forced_boundary = int(forced_boundary)
+    a.mass_partial_len = int(mass_partial_prev.shape[-1]) if mass_partial_prev is not None else 0
+    a.mass_row_count = int(mass_row_count)
+    a.q_delta = _ptr(q_delta)
+    a.mass_partial_prev = _ptr(mass_partial_prev)
+    a.state = _ptr(state)
+    a.mode_out = _ptr(mode_out)
+    a.gbar_out = _ptr(gbar_out)
+    a.m_out = _ptr(m_out)
+    return check("refadapt_gate", _lib.load().refadapt_gate(ctypes.byref(a), _stream(stream)))
+
+
+def refadapt_ref_cache_update(k_src, v_src, k_cache, v_cache, mode, t, a_b=None, x_src=None, x_cache=None,
+                              stream=None):
+    lib = _lib.load()
+    B, H, _, d = k_src.shape
+    ks, vs, kc, vc = seg(k_src), seg(v_src), seg(k_cache), seg(v_cache)
+    if x_src is not None:
+        xs, xc = seg(x_src), seg(x_cache)
+        xp, xcp = ctypes.byref(xs), ctypes.byref(xc)
+        x_heads, x_width = x_src.shape[1], x_src.shape[3]
+    else:
+        xp = xcp = None
+        x_heads = x_width = 0
+    return check("refadapt_ref_cache_update", lib.refadapt_ref_cache_update(
+        ctypes.byref(ks), ctypes.byref(vs), ctypes.byref(kc), ctypes.byref(vc), B, H, d, xp, xcp,
+        x_heads, x_width, _ptr(mode), int(t), _ptr(a_b), _stream(stream)))
+
+
+def refadapt_set_wait_budget_ns(ns):
+    _lib.load().refadapt_set_wait_budget_ns(int(ns))
+
+
+def refadapt_check_error(err_word, stream=None):
+    return check("refadapt_check_error", _lib.load().refadapt_check_error(_ptr(err_word), _stream(stream)))
+
+
+def refadapt_selftest_wait_timeout(err_word, budget_ns, stream=None):
+    return check("refadapt_selftest_wait_timeout",
+                 _lib.load().refadapt_selftest_wait_timeout(_ptr(err_word), int(budget_ns), _stream(stream)))
+
+
+def refadapt_version() -> int:
+    return int(_lib.load().refadapt_version())

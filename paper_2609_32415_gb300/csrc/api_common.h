@@ -1,0 +1,32 @@
+// Host-side helpers shared by the C-ABI entry points: argument checks, the
+// thread-local error message, device properties and the wait budget.
+#pragma once
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "refadapt.h"
+
+namespace ra {
+
+// Records a one-line reason for the last RA_EINVAL / RA_ECUDA of this thread.
+void set_error(const char* fmt, ...);
+void clear_error();
+
+uint64_t wait_budget_ns();
+int num_sms();  // of the current device (cached per device)
+
+// A bf16 segment usable by 16-byte vector access and by TMA: 16-byte aligned
+// pointer and strides, n >= 0, non-negative strides. `what` names it in errors.
+bool check_seg(const ra_seg& s, const char* what, bool allow_null_if_empty = true);
+
+inline ra_status launch_status(const char* what) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    set_error("%s: launch failed: %s", what, cudaGetErrorString(e));
+    return RA_ECUDA;
+  }
+  return RA_OK;
+}
+
+}  // namespace ra

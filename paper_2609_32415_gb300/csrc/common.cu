@@ -1,0 +1,138 @@
+// Status strings, error message, wait budget and the error-word check.
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <cstdarg>
+#include <cstdio>
+#include <mutex>
+
+#include "api_common.h"
+#include "tc_ptx.cuh"
+
+namespace ra {
+
+namespace {
+thread_local char g_err[512] = {0};
+std::atomic<uint64_t> g_budget_ns{2000000000ull};
+std::mutex g_sm_mu;
+int g_sm_count[64] = {0};
+}  // namespace
+
+void set_error(const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+}
+void clear_error() { g_err[0] = 0; }
+
+uint64_t wait_budget_ns() { return g_budget_ns.load(std::memory_order_relaxed); }
+
+int num_sms() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 148;
+  if (dev < 0 || dev >= 64) dev = 0;
+  std::lock_guard<std::mutex> lk(g_sm_mu);
+  if (g_sm_count[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 148;
+    g_sm_count[dev] = n;
+  }
+  return g_sm_count[dev];
+}
+
+bool check_seg(const ra_seg& s, const char* what, bool allow_null_if_empty) {
+  if (s.n < 0) {
+    set_error("%s: n = %d is negative", what, s.n);
+    return false;
+  }
+  if (s.ptr == nullptr) {
+    if (s.n == 0 && allow_null_if_empty) return true;
+    set_error("%s: ptr is NULL", what);
+    return false;
+  }
+  if (reinterpret_cast<uintptr_t>(s.ptr) % 16 != 0) {
+    set_error("%s: ptr is not 16-byte aligned", what);
+    return false;
+  }
+  if (s.stride_b < 0 || s.stride_h < 0 || s.stride_n < 0) {
+    set_error("%s: negative stride", what);
+    return false;
+  }
+  if (s.stride_b % 8 || s.stride_h % 8 || s.stride_n % 8) {
+    set_error("%s: strides must be multiples of 8 elements (16 bytes)", what);
+    return false;
+  }
+  return true;
+}
+
+}  // namespace ra
+
+extern "C" const char* refadapt_status_string(ra_status s) {
+  switch (s) {
+    case RA_OK: return "RA_OK";
+    case RA_EINVAL: return "RA_EINVAL: invalid argument";
+    case RA_EUNSUPPORTED: return "RA_EUNSUPPORTED: unsupported configuration";
+    case RA_ECUDA: return "RA_ECUDA: CUDA error";
+    case RA_ETIMEOUT: return "RA_ETIMEOUT: device wait ran out of its budget";
+  }
+  return "unknown ra_status";
+}
+
+extern "C" const char* refadapt_last_error(void) { return ra::g_err; }
+
+extern "C" void refadapt_set_wait_budget_ns(uint64_t ns) {
+  ra::g_budget_ns.store(ns == 0 ? 1 : ns, std::memory_order_relaxed);
+}
+
+extern "C" ra_status refadapt_check_error(int32_t* err_word, void* stream) {
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (cudaStreamSynchronize(st) != cudaSuccess) {
+    ra::set_error("refadapt_check_error: %s", cudaGetErrorString(cudaGetLastError()));
+    return RA_ECUDA;
+  }
+  if (err_word == nullptr) return RA_OK;
+  int32_t host = 0;
+  if (cudaMemcpy(&host, err_word, sizeof(host), cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemset(err_word, 0, sizeof(int32_t)) != cudaSuccess) {
+    ra::set_error("refadapt_check_error: %s", cudaGetErrorString(cudaGetLastError()));
+    return RA_ECUDA;
+  }
+  if (host & 1) {
+    ra::set_error("a device-side wait exceeded its budget");
+    return RA_ETIMEOUT;
+  }
+  return RA_OK;
+}
+
+extern "C" int32_t refadapt_version(void) { return 1; }
+
+namespace ra {
+namespace {
+__global__ void selftest_wait_kernel(int32_t* err, uint64_t budget_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const WaitCtl ctl{&abort_flag, err, budget_ns};
+    (void)mbar_wait(&bar, 0, ctl);  // nothing arrives: returns false after budget_ns
+  }
+}
+}  // namespace
+}  // namespace ra
+
+extern "C" ra_status refadapt_selftest_wait_timeout(int32_t* err_word, uint64_t budget_ns, void* stream) {
+  ra::clear_error();
+  if (!err_word) {
+    ra::set_error("refadapt_selftest_wait_timeout: err_word is NULL");
+    return RA_EINVAL;
+  }
+  if (budget_ns > 1000000000ull) budget_ns = 1000000000ull;
+  ra::selftest_wait_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(err_word, budget_ns);
+  return ra::launch_status("refadapt_selftest_wait_timeout");
+}

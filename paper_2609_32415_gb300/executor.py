@@ -1,0 +1,105 @@
+"""Algorithm 1's host loop over the C ABI: one denoising step = for each block,
+Q change -> gate -> cache materialisation -> joint attention, all enqueued on
+one stream with the decisions kept on the device (no host sync inside a step).
+
+Per block b the executor owns the cache state of paper Eq. 11: reference K and
+V, the cached reference hidden state (here the reference query, which is what
+restoring the hidden state at a boundary produces in this hot path) and a_b.
+The joint-attention kernel always reads reference Q/K/V from that cache slot:
+COMPUTE / FULL blocks refresh the slot first (so they see fresh values),
+REUSE and BOUNDARY blocks see the values of the last materialisation.
+"""
+import torch
+
+from . import api
+from ._lib import RA_MODE_BOUNDARY, RA_MODE_COMPUTE, RA_MODE_FULL, RA_MODE_REUSE  # noqa: F401
+
+ROLES = ("text", "ref", "tgt")
+
+
+def roles_from_joint(X, offsets, n):
+    """Role views of a joint tensor X[3, B, H, N, d] (q, k, v stacked).
+
+    Returns dict role -> (q, k, v), each a [B, H, n_role, d] view."""
+    out = {}
+    for r in ROLES:
+        o, k = offsets[r], n[r]
+        out[r] = (X[0, :, :, o:o + k, :], X[1, :, :, o:o + k, :], X[2, :, :, o:o + k, :])
+    return out
+
+
+class Executor:
+    def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
+                 mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
+                 device="cuda"):
+        self.n_blocks, self.B, self.H, self.d = n_blocks, B, H, d
+        self.n = {"text": n_text, "ref": n_ref, "tgt": n_tgt}
+        self.theta, self.delta_max, self.eps = float(theta), int(delta_max), float(eps)
+        self.mass_rows, self.forced_boundary = int(mass_rows), int(forced_boundary)
+        self.softmax_scale = float(softmax_scale)
+        dev = torch.device(device)
+        self.bias = None if bias is None else torch.as_tensor(bias, dtype=torch.float32, device=dev).contiguous()
+        shape = (n_blocks, B, H, n_ref, d)
+        self.cache_k = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+        self.cache_v = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+        self.cache_x = torch.zeros(shape, dtype=torch.bfloat16, device=dev)
+        self.a_b = torch.full((n_blocks, B), -1, dtype=torch.int32, device=dev)
+        self.mpl = api.refadapt_mass_partial_len(n_text, n_tgt)
+        self.mass = torch.zeros((n_blocks, B, H, self.mpl), dtype=torch.float32, device=dev)
+        self.mass_row_count = n_tgt + (n_text if mass_rows == 1 else 0)
+        self.D = torch.zeros((n_blocks, B, H), dtype=torch.float32, device=dev)
+        self.log_steps = int(log_steps)
+        self.modes = torch.full((self.log_steps, n_blocks, B), -1, dtype=torch.int32, device=dev)
+        self.gbar = torch.zeros((self.log_steps, n_blocks, B), dtype=torch.float32, device=dev)
+        self.M = torch.zeros((self.log_steps, n_blocks, B, H), dtype=torch.float32, device=dev)
+        self.workspace = api.q_delta_workspace(B, H, dev)
+        self.state = api.new_state(B, dev)
+        self.err = torch.zeros(1, dtype=torch.int32, device=dev)
+        self._prev_qtgt = [None] * n_blocks
+        self._out = None
+
+    def scratch_outputs(self):
+        """One shared set of O buffers (text, ref, tgt) reused by every block."""
+        if self._out is None:
+            self._out = {r: torch.empty((self.B, self.H, self.n[r], self.d), dtype=torch.bfloat16,
+                                        device=self.cache_k.device) for r in ROLES}
+        return self._out
+
+    def block(self, t, b, x, out, log_index=None, stream=None):
+        """Enqueue block b of step t. x: dict role -> (q, k, v) [B, H, n, d] views;
+        out: dict role -> O [B, H, n, d]."""
+        li = (t % self.log_steps) if log_index is None else log_index
+        mode = self.modes[li, b]
+        qt = x["tgt"][0]
+        have_prev = t >= 1 and self._prev_qtgt[b] is not None
+        if have_prev:
+            api.refadapt_q_delta(qt, self._prev_qtgt[b], self.D[b], self.workspace, self.eps, stream)
+        api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
+                          q_delta=self.D[b] if have_prev else None,
+                          mass_partial_prev=self.mass[b] if have_prev else None,
+                          mass_row_count=self.mass_row_count, forced_boundary=self.forced_boundary,
+                          gbar_out=self.gbar[li, b], m_out=self.M[li, b], stream=stream)
+        qr, kr, vr = x["ref"]
+        api.refadapt_ref_cache_update(kr, vr, self.cache_k[b], self.cache_v[b], mode, t, self.a_b[b],
+                                      x_src=qr, x_cache=self.cache_x[b], stream=stream)
+        api.refadapt_joint_attn(
+            (x["text"][0], self.cache_x[b], qt),
+            (x["text"][1], self.cache_k[b], x["tgt"][1]),
+            (x["text"][2], self.cache_v[b], x["tgt"][2]),
+            (out["text"], out["ref"], out["tgt"]),
+            self.mass[b], mode=mode, softmax_scale=self.softmax_scale, ref_logit_bias=self.bias,
+            mass_rows=self.mass_rows, err_word=self.err, stream=stream)
+        self._prev_qtgt[b] = qt
+
+    def step(self, t, inputs, outs=None, log_index=None, stream=None, after_block=None):
+        """Enqueue one denoising step. inputs[b]: dict role -> (q, k, v);
+        outs[b] (optional): dict role -> O. The caller keeps step t's target Q
+        alive until step t + 1 has been enqueued (it is read as q_{t-1})."""
+        for b in range(self.n_blocks):
+            out = outs[b] if outs is not None else self.scratch_outputs()
+            self.block(t, b, inputs[b], out, log_index, stream)
+            if after_block is not None:
+                after_block(t, b)
+
+    def check(self, stream=None):
+        api.refadapt_check_error(self.err, stream)

@@ -1,0 +1,113 @@
+"""Closed-loop parity: Algorithm 1 run by the Executor over the C ABI against the
+oracle's closed loop on the same seeded bf16 inputs (modes, D, M, O)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from _helpers import D_REL, M_ABS, TIE_BAND, bits, o_close
+
+pytestmark = pytest.mark.gpu
+
+ROLES = ("text", "ref", "tgt")
+
+
+def _run_both(wl, o_sample=None):
+    from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
+    traj = synth.Trajectory(wl, device="cuda")
+    ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max,
+                  wl.eps, mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
+                  log_steps=wl.n_steps)
+    keep, outs, D = {}, {}, np.zeros((wl.n_steps, wl.n_blocks, wl.B, wl.H))
+    for t in range(wl.n_steps):
+        xs, os_ = [], []
+        for b in range(wl.n_blocks):
+            X = traj.get(t, b)
+            keep[(t, b)] = X
+            xs.append(roles_from_joint(X, wl.offsets(), wl.n))
+            os_.append({r: torch.full((wl.B, wl.H, wl.n[r], wl.d), float("nan"), dtype=torch.bfloat16,
+                                      device="cuda") for r in ROLES})
+
+        def grab(tt, bb):
+            D[tt, bb] = ex.D[bb].double().cpu().numpy()
+
+        ex.step(t, xs, os_, after_block=grab)
+        outs[t] = os_
+    torch.cuda.synchronize()
+    ex.check()
+    modes = ex.modes.cpu().numpy()
+    gbar = ex.gbar.double().cpu().numpy()
+    Mlog = ex.M.double().cpu().numpy()
+
+    def raw(t, b):
+        X = keep[(t, b)]
+        off = wl.offsets()
+        return {r: tuple(bits(X[z, :, :, off[r]:off[r] + wl.n[r], :]) for z in range(3)) for r in ROLES}
+
+    def tie(t, b, s):
+        return modes[t, b, s] == 1
+
+    rec = oracle.closed_loop(raw, wl.n_steps, wl.n_blocks, wl.B, theta=wl.theta, delta_max=wl.delta_max,
+                             eps=wl.eps, bias=wl.bias, mass_rows=wl.mass_rows,
+                             forced_boundary=wl.forced_boundary, tie=tie, o_rows=o_sample)
+    return modes, gbar, Mlog, D, outs, rec
+
+
+def _compare(wl, modes, gbar, Mlog, D, outs, rec, o_sample=None):
+    ties = 0
+    for t in range(wl.n_steps):
+        for b in range(wl.n_blocks):
+            r = rec[t][b]
+            assert list(modes[t, b]) == r["mode"], (t, b, modes[t, b], r["mode"])
+            for s in range(wl.B):
+                if np.isfinite(r["gbar"][s]) and abs(r["gbar"][s] - wl.theta) < TIE_BAND:
+                    ties += 1
+            if t >= 1:
+                rel = np.abs(D[t, b] - r["D"]) / np.abs(r["D"])
+                assert rel.max() <= D_REL, (t, b, rel.max())
+                np.testing.assert_allclose(gbar[t, b], r["gbar"], rtol=1e-4, atol=1e-6)
+            if t + 1 < wl.n_steps:
+                dm = np.abs(Mlog[t + 1, b] - r["M"]).max()
+                assert dm <= M_ABS, (t, b, dm)
+            for s in range(wl.B):
+                for role in ROLES:
+                    ref = r["O"][s][role]
+                    got = outs[t][b][role][s]
+                    if ref is None:
+                        assert torch.isnan(got.float()).all()
+                        continue
+                    g = got.double().cpu().numpy()
+                    if o_sample is not None:
+                        g = g[:, o_sample(t, b, s)[role], :]
+                    ok, worst, nw = o_close(g, ref)
+                    assert ok, (t, b, s, role, worst, nw)
+    return ties
+
+
+@pytest.mark.parametrize("theta", [0.05, 0.1, 0.2])
+def test_closed_loop_single_block_workload(cuda_ok, theta):
+    from paper_2609_32415_gb300 import synth
+    wl = synth.make_workload("c1", theta=theta)
+    res = _run_both(wl)
+    _compare(wl, *res)
+
+
+def test_closed_loop_multi_block_depth_profile(cuda_ok):
+    """Five blocks, B=2, ragged segments, increasing target drift with depth so
+    the boundary moves; delta_max=3 forces a full refresh mid-trajectory."""
+    from paper_2609_32415_gb300 import synth
+    wl = synth.custom_workload(2, 4, 128, 33, 300, 200, n_blocks=5, n_steps=6, ref_drift=0.05,
+                               tgt_drift=[0.05, 0.1, 0.2, 0.3, 0.4], theta=0.08, delta_max=3)
+    res = _run_both(wl)
+    _compare(wl, *res)
+    modes = res[0]
+    assert (modes == 0).any() and (modes == 1).any() and (modes == 2).any() and (modes == 3).any()
+
+
+def test_closed_loop_forced_boundary_and_bias(cuda_ok):
+    from paper_2609_32415_gb300 import synth
+    wl = synth.custom_workload(1, 3, 64, 16, 260, 140, n_blocks=4, n_steps=3, theta=float("inf"),
+                               delta_max=8, forced_boundary=2, bias=[-3.0, -1.0, 0.0], mass_rows=1)
+    res = _run_both(wl)
+    _compare(wl, *res)
+    assert list(res[0][1, :, 0]) == [0, 0, 1, 2]
