@@ -57,6 +57,7 @@ class Executor:
         self.err = torch.zeros(1, dtype=torch.int32, device=dev)
         self._prev_qtgt = [None] * n_blocks
         self._out = None
+        self.attn_hook = None   # optional callable(phase in {"pre", "post"}, t, b), e.g. CUDA events
 
     def scratch_outputs(self):
         """One shared set of O buffers (text, ref, tgt) reused by every block."""
@@ -82,6 +83,8 @@ class Executor:
         qr, kr, vr = x["ref"]
         api.refadapt_ref_cache_update(kr, vr, self.cache_k[b], self.cache_v[b], mode, t, self.a_b[b],
                                       x_src=qr, x_cache=self.cache_x[b], stream=stream)
+        if self.attn_hook is not None:
+            self.attn_hook("pre", t, b)
         api.refadapt_joint_attn(
             (x["text"][0], self.cache_x[b], qt),
             (x["text"][1], self.cache_k[b], x["tgt"][1]),
@@ -89,6 +92,8 @@ class Executor:
             (out["text"], out["ref"], out["tgt"]),
             self.mass[b], mode=mode, softmax_scale=self.softmax_scale, ref_logit_bias=self.bias,
             mass_rows=self.mass_rows, err_word=self.err, stream=stream)
+        if self.attn_hook is not None:
+            self.attn_hook("post", t, b)
         self._prev_qtgt[b] = qt
 
     def step(self, t, inputs, outs=None, log_index=None, stream=None, after_block=None):
