@@ -374,24 +374,26 @@ def time_e2e(wl, inputs, warmup, steps):
     return {"value": ms / steps, "unit": "ms/step", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
 
 
-def time_q_delta(wl, inputs, reps=50):
-    """HBM roofline of the Q-change reduction alone, on one block's target Q."""
+def time_q_delta(wl, inputs, reps=48):
+    """HBM roofline of the Q-change reduction alone: target Q of step 1 vs step
+    0, rotating over 8 blocks (8 x 50 MB > L2, so every launch reads HBM)."""
     import torch
     from paper_2609_32415_gb300 import api, roles_from_joint
-    a = roles_from_joint(inputs[1][0], wl.offsets(), wl.n)["tgt"][0]
-    b = roles_from_joint(inputs[0][0], wl.offsets(), wl.n)["tgt"][0]
+    nb = min(8, wl.n_blocks)
+    pairs = [(roles_from_joint(inputs[1][b], wl.offsets(), wl.n)["tgt"][0],
+              roles_from_joint(inputs[0][b], wl.offsets(), wl.n)["tgt"][0]) for b in range(nb)]
     ws = api.q_delta_workspace(wl.B, wl.H)
     out = torch.empty((wl.B, wl.H), dtype=torch.float32, device="cuda")
-    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
     times = []
-    for i in range(reps + 3):
-        flush.fill_(float(i))                  # evict L2 between launches
+    for i in range(reps + nb):
+        a, b = pairs[i % nb]
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda._sleep(200000)   # keep the stream busy so e0 -> launch -> e1 are queued back to back
         e0.record()
         api.refadapt_q_delta(a, b, out, ws, wl.eps)
         e1.record()
         torch.cuda.synchronize()
-        if i >= 3:
+        if i >= nb:
             times.append(e0.elapsed_time(e1))
     byts = 4 * wl.n_tgt * wl.H * wl.d * wl.B
     ms = statistics.median(times)

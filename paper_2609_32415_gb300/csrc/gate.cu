@@ -25,7 +25,7 @@ namespace ra {
 namespace gate {
 
 constexpr int32_t kMagic = 0x52414701;
-constexpr int THREADS = 128;
+constexpr int THREADS = 256;
 
 struct Params {
   double theta;
@@ -50,13 +50,17 @@ __global__ void init_kernel(ra_state* st, int32_t B) {
   }
 }
 
-// One CTA: thread s handles sample s (loop if B > THREADS). Sums run in a
-// fixed order in fp64.
+// One CTA. Warps compute M_{t-1,b,h} for every (sample, head) from the mass
+// partials (lane-strided sums, then a butterfly: fixed order, fp64) into
+// shared memory; then thread s takes sample s through the decision.
 __global__ void __launch_bounds__(THREADS) gate_kernel(const Params p) {
+  extern __shared__ double m_sh[];  // [B * H]
   ra_state* st = p.st;
   int32_t* reactivated = reinterpret_cast<int32_t*>(st + 1);
   int32_t* boundary = reactivated + p.B;
   __shared__ int32_t full_step;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nwarps = THREADS / 32;
   if (threadIdx.x == 0) {
     if (p.b == 0) {
       if (p.t == 0) {
@@ -72,25 +76,30 @@ __global__ void __launch_bounds__(THREADS) gate_kernel(const Params p) {
     }
     full_step = st->full_step;
   }
+  for (int sh = warp; sh < p.B * p.H; sh += nwarps) {
+    double acc = 0.0;
+    if (p.mp) {
+      const float* row = p.mp + int64_t(sh) * p.mpl;
+      for (int i = lane; i < p.mpl; i += 32) acc += double(row[i]);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    }
+    if (lane == 0) {
+      const double m = acc / double(p.mass_rows_count);
+      m_sh[sh] = m;
+      if (p.m_out && p.mp) p.m_out[sh] = float(m);
+    }
+  }
   __syncthreads();
   for (int s = threadIdx.x; s < p.B; s += blockDim.x) {
     if (p.b == 0) {
       reactivated[s] = 0;
       boundary[s] = -1;
     }
-    double gsum = 0.0;
     const bool have = (p.t >= 1) && p.qd && p.mp;
-    for (int h = 0; h < p.H; ++h) {
-      double m = 0.0;
-      if (p.mp) {
-        const float* row = p.mp + (int64_t(s) * p.H + h) * p.mpl;
-        double acc = 0.0;
-        for (int i = 0; i < p.mpl; ++i) acc += double(row[i]);
-        m = acc / double(p.mass_rows_count);
-        if (p.m_out) p.m_out[s * p.H + h] = float(m);
-      }
-      if (have) gsum += double(p.qd[s * p.H + h]) * m;
-    }
+    double gsum = 0.0;
+    if (have)
+      for (int h = 0; h < p.H; ++h) gsum += double(p.qd[s * p.H + h]) * m_sh[s * p.H + h];
     const double gbar = have ? gsum / double(p.H) : NAN;
     if (p.gbar_out) p.gbar_out[s] = float(gbar);
     int32_t mode;
@@ -154,6 +163,10 @@ extern "C" ra_status refadapt_gate(const ra_gate_args* a, void* stream) {
     set_error("refadapt_gate: mass_partial_len and mass_row_count must be >= 1");
     return RA_EINVAL;
   }
+  if (int64_t(a->B) * a->H > 6144) {
+    set_error("refadapt_gate: B * H must be <= 6144");
+    return RA_EINVAL;
+  }
   if (std::isnan(a->theta)) {
     set_error("refadapt_gate: theta is NaN");
     return RA_EINVAL;
@@ -174,6 +187,7 @@ extern "C" ra_status refadapt_gate(const ra_gate_args* a, void* stream) {
   p.mode_out = a->mode_out;
   p.gbar_out = a->gbar_out;
   p.m_out = a->m_out;
-  gate::gate_kernel<<<1, gate::THREADS, 0, static_cast<cudaStream_t>(stream)>>>(p);
+  const size_t sh_bytes = size_t(a->B) * a->H * sizeof(double);
+  gate::gate_kernel<<<1, gate::THREADS, sh_bytes, static_cast<cudaStream_t>(stream)>>>(p);
   return launch_status("refadapt_gate");
 }

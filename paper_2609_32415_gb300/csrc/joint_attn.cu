@@ -1,25 +1,30 @@
 // refadapt_joint_attn: joint [text; reference; target] attention with the
 // per-tile reference mass, on tcgen05 tensor cores (sm_103a).
 //
-// One CTA computes one 128-row Q tile of one role for one (sample, head):
-//   warp 0      TMA producer: the Q tile once, then K and V tiles of the text,
-//               reference (cache slot) and target segments in that order,
+// One CTA computes a pair of 128-row Q tiles (A, B) of one role for one
+// (sample, head); both tiles share every K/V tile it streams:
+//   warp 0      TMA producer: Q tiles A and B once, then K and V tiles of the
+//               text, reference (cache slot) and target segments in that order
 //               into a STAGES-deep ring of 128-byte-swizzled shared buffers.
-//   warp 1      TMEM allocator and MMA issuer (one thread): S_j = Q K_j^T into
-//               one of two TMEM S buffers (kind::f16, fp32 accumulate), then
-//               O += P_j V_j with P_j read from TMEM (it overwrites the first
-//               64 columns of S_j as packed bf16). S_{j+1} is issued before
-//               O += P_j V_j so the tensor core works while softmax j runs.
-//   warps 2..5  softmax / epilogue: thread = query row = TMEM lane. Online
-//               softmax in log2 units with a lazy rescale (the running max is
-//               only moved when a tile's max exceeds it by more than 2^8), the
-//               row sum l and the reference-only row sum l_ref (paper Eq. 4's
-//               inner sum is l_ref / l), then O / l -> bf16 global, and the
-//               tile's sum of l_ref / l over mass rows -> mass_partial.
-// Segment tails: TMA zero-fills rows past a segment's end; the softmax masks
-// those key columns to probability 0 and the epilogue skips those query rows.
-// Every mbarrier wait is bounded (WaitCtl); on a timeout the CTA drains its own
-// TMA and MMA work, frees TMEM, flags the caller's error word and returns.
+//   warp 1      TMEM allocator and MMA issuer (one thread). TMEM columns:
+//               S_A [0,128), S_B [128,256), O_A [256,..), O_B [384,..).
+//               S_t = Q_t K_j^T (kind::f16, fp32 accumulate); P_t is written
+//               back over the first 64 columns of S_t as packed bf16 and read
+//               from TMEM as the A operand of O_t += P_t V_j. Issue order per
+//               key tile: PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1), so the tensor
+//               core works on one tile while the other tile's softmax runs.
+//   warps 2..5  softmax / epilogue of tile A, warps 6..9 of tile B: thread =
+//               query row = TMEM lane (lane quarter = warp % 4). Online softmax
+//               in log2 units with a lazy rescale (the running max only moves
+//               when a tile's max exceeds it by more than 2^8), the row sum l
+//               and the reference-only row sum l_ref (paper Eq. 4's inner sum
+//               is l_ref / l); then O / l -> bf16 global and the tile's sum of
+//               l_ref / l over its mass rows -> mass_partial.
+// Segment tails: TMA zero-fills rows past a segment's end; tail key tiles mask
+// the padded columns to -inf (probability 0) and the epilogue skips padded
+// query rows. Every mbarrier wait is bounded (WaitCtl); on a timeout the CTA
+// drains its own TMA and MMA work, frees TMEM, flags the caller's error word
+// and returns.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 #include <cuda_bf16.h>
@@ -38,7 +43,7 @@ namespace attn {
 
 constexpr int BM = 128;  // query rows per tile (= TMEM lanes)
 constexpr int BN = 128;  // keys per tile
-constexpr int NUM_THREADS = 192;
+constexpr int NUM_THREADS = 320;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleThresh = 8.0f;  // log2 units: p <= 2^8 between rescales
 
@@ -46,23 +51,23 @@ template <int D>
 struct Cfg {
   static constexpr int CHUNKS = D / 64;           // 64-element (128-byte) swizzle chunks per row
   static constexpr int CHUNK_BYTES = BM * 128;    // one chunk of a 128-row tile
-  static constexpr int TILE_BYTES = BM * D * 2;   // Q, K or V tile (BN == BM)
+  static constexpr int TILE_BYTES = BM * D * 2;   // one Q, K or V tile (BN == BM)
   static constexpr int STAGES = (D == 128) ? 2 : 4;
-  static constexpr int OFF_Q = 0;
-  static constexpr int OFF_K = OFF_Q + TILE_BYTES;
+  static constexpr int OFF_Q = 0;                 // Q tiles A and B
+  static constexpr int OFF_K = OFF_Q + 2 * TILE_BYTES;
   static constexpr int OFF_V = OFF_K + STAGES * TILE_BYTES;
   static constexpr int OFF_BAR = OFF_V + STAGES * TILE_BYTES;
-  // q_full, k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_ready[2], o_done, drain
-  static constexpr int NUM_BARS = 1 + 4 * STAGES + 2 + 2 + 1 + 1;
-  static constexpr int OFF_MISC = OFF_BAR + NUM_BARS * 8;  // tmem slot, abort flag, 4 floats
+  // q_full, k_full[S], k_empty[S], v_full[S], v_empty[S], s_full[2], p_ready[2], o_done[2], drain
+  static constexpr int NUM_BARS = 1 + 4 * STAGES + 2 + 2 + 2 + 1;
+  static constexpr int OFF_MISC = OFF_BAR + NUM_BARS * 8;  // tmem slot, abort flag, 8 floats
   static constexpr int SMEM_BYTES = OFF_MISC + 64;
   static constexpr int SMEM_ALLOC = SMEM_BYTES + 1024;  // slack for 1024-byte alignment
   static constexpr uint32_t TMEM_COLS = 512;
-  static constexpr uint32_t TM_S0 = 0, TM_S1 = 128, TM_O = 256;
+  static constexpr uint32_t TM_S = 0, TM_O = 256;       // + 128 * tile
   static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 };
 
-struct alignas(64) Params {
+struct Params {
   CUtensorMap tm_q[3];
   CUtensorMap tm_k[3];
   CUtensorMap tm_v[3];
@@ -70,6 +75,7 @@ struct alignas(64) Params {
   int64_t o_sb[3], o_sh[3], o_sn[3];
   int32_t n[3];
   int32_t q_tiles[3];
+  int32_t q_blocks[3];  // pairs of Q tiles
   int32_t kv_tiles[3];
   int32_t B, H;
   int32_t mass_rows;
@@ -95,23 +101,87 @@ __device__ __forceinline__ void kv_tile(const Params& p, int j, int& r, int& row
   }
 }
 
+// Row maximum over the 64 logits in v[] (columns col0 .. col0+63 of the tile);
+// TAIL ignores columns >= nvalid.
+template <bool TAIL>
+__device__ __forceinline__ float max64(const float (&v)[64], int col0, int nvalid, float m_in) {
+  float m0 = m_in, m1 = -INFINITY, m2 = -INFINITY, m3 = -INFINITY;
+#pragma unroll
+  for (int c = 0; c < 64; c += 8) {
+    if (TAIL) {
+      const int e = col0 + c;
+      m0 = fmax3f(m0, (e < nvalid) ? v[c] : -INFINITY, (e + 1 < nvalid) ? v[c + 1] : -INFINITY);
+      m1 = fmax3f(m1, (e + 2 < nvalid) ? v[c + 2] : -INFINITY, (e + 3 < nvalid) ? v[c + 3] : -INFINITY);
+      m2 = fmax3f(m2, (e + 4 < nvalid) ? v[c + 4] : -INFINITY, (e + 5 < nvalid) ? v[c + 5] : -INFINITY);
+      m3 = fmax3f(m3, (e + 6 < nvalid) ? v[c + 6] : -INFINITY, (e + 7 < nvalid) ? v[c + 7] : -INFINITY);
+    } else {
+      m0 = fmax3f(m0, v[c], v[c + 1]);
+      m1 = fmax3f(m1, v[c + 2], v[c + 3]);
+      m2 = fmax3f(m2, v[c + 4], v[c + 5]);
+      m3 = fmax3f(m3, v[c + 6], v[c + 7]);
+    }
+  }
+  return fmaxf(fmaxf(m0, m1), fmaxf(m2, m3));
+}
+
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
+  tmem_ld32(taddr, *reinterpret_cast<uint32_t(*)[32]>(&v[0]));
+  tmem_ld32(taddr + 32, *reinterpret_cast<uint32_t(*)[32]>(&v[32]));
+  tmem_ld_wait();
+}
+
+// Probabilities of 64 logits (columns col0 ..), p = 2^(v * sl2 + negm), packed
+// to bf16 into 32 TMEM columns at p_taddr. Returns their fp32 sum. TAIL masks
+// columns >= nvalid to probability 0.
+template <bool TAIL>
+__device__ __forceinline__ float exp64_store(const float (&v)[64], int col0, int nvalid, uint64_t scale2,
+                                             uint64_t off2, uint32_t p_taddr) {
+  uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
+  uint32_t pk[32];
+#pragma unroll
+  for (int c = 0; c < 64; c += 4) {
+    float a0, a1, b0, b1;
+    f2_unpack(f2_fma(f2_pack(v[c], v[c + 1]), scale2, off2), a0, a1);
+    f2_unpack(f2_fma(f2_pack(v[c + 2], v[c + 3]), scale2, off2), b0, b1);
+    float p0 = ex2_approx(a0), p1 = ex2_approx(a1), p2 = ex2_approx(b0), p3 = ex2_approx(b1);
+    if (TAIL) {
+      const int e = col0 + c;
+      p0 = (e < nvalid) ? p0 : 0.f;
+      p1 = (e + 1 < nvalid) ? p1 : 0.f;
+      p2 = (e + 2 < nvalid) ? p2 : 0.f;
+      p3 = (e + 3 < nvalid) ? p3 : 0.f;
+    }
+    acc0 = f2_add(acc0, f2_pack(p0, p1));
+    acc1 = f2_add(acc1, f2_pack(p2, p3));
+    pk[c / 2] = pack_bf16x2(p0, p1);
+    pk[c / 2 + 1] = pack_bf16x2(p2, p3);
+  }
+  tmem_st32(p_taddr, pk);
+  float s0, s1, s2, s3;
+  f2_unpack(acc0, s0, s1);
+  f2_unpack(acc1, s2, s3);
+  return (s0 + s1) + (s2 + s3);
+}
+
 template <int D>
 __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid_constant__ Params p) {
   using C = Cfg<D>;
   constexpr int S = C::STAGES;
   const int b = blockIdx.z, h = blockIdx.y;
-  int qt = blockIdx.x, role;
-  if (qt < p.q_tiles[0]) {
+  int qb = blockIdx.x, role;
+  if (qb < p.q_blocks[0]) {
     role = 0;
-  } else if (qt - p.q_tiles[0] < p.q_tiles[1]) {
-    qt -= p.q_tiles[0];
+  } else if (qb - p.q_blocks[0] < p.q_blocks[1]) {
+    qb -= p.q_blocks[0];
     role = 1;
   } else {
-    qt -= p.q_tiles[0] + p.q_tiles[1];
+    qb -= p.q_blocks[0] + p.q_blocks[1];
     role = 2;
   }
   const int mode = p.mode ? __ldg(p.mode + b) : int(RA_MODE_FULL);
   if (role == 1 && mode == RA_MODE_REUSE) return;  // reference rows skipped (uniform exit)
+  const int tileA = 2 * qb;
+  const bool has_b = (tileA + 1) < p.q_tiles[role];
 
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
@@ -121,13 +191,13 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
   uint64_t* k_empty = bars + 1 + S;
   uint64_t* v_full = bars + 1 + 2 * S;
   uint64_t* v_empty = bars + 1 + 3 * S;
-  uint64_t* s_full = bars + 1 + 4 * S;
-  uint64_t* p_ready = bars + 3 + 4 * S;
-  uint64_t* o_done = bars + 5 + 4 * S;
-  uint64_t* drain = bars + 6 + 4 * S;
+  uint64_t* s_full = bars + 1 + 4 * S;   // [tile]
+  uint64_t* p_ready = bars + 3 + 4 * S;  // [tile]
+  uint64_t* o_done = bars + 5 + 4 * S;   // [tile]
+  uint64_t* drain = bars + 7 + 4 * S;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + C::OFF_MISC);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + C::OFF_MISC + 4);
-  float* red = reinterpret_cast<float*>(smem + C::OFF_MISC + 16);
+  float* red = reinterpret_cast<float*>(smem + C::OFF_MISC + 16);  // [tile][quarter]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
@@ -138,11 +208,11 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
       mbar_init(v_full + s, 1);
       mbar_init(v_empty + s, 1);
     }
-    mbar_init(s_full, 1);
-    mbar_init(s_full + 1, 1);
-    mbar_init(p_ready, 128);
-    mbar_init(p_ready + 1, 128);
-    mbar_init(o_done, 1);
+    for (int t = 0; t < 2; ++t) {
+      mbar_init(s_full + t, 1);
+      mbar_init(p_ready + t, 128);
+      mbar_init(o_done + t, 1);
+    }
     mbar_init(drain, 1);
     *abort_flag = 0;
     fence_mbar_init();
@@ -164,11 +234,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
           tma_prefetch_desc(&p.tm_k[r]);
           tma_prefetch_desc(&p.tm_v[r]);
         }
-      int k_issued[S], v_issued[S];
-      for (int s = 0; s < S; ++s) k_issued[s] = v_issued[s] = 0;
-      mbar_arrive_expect_tx(q_full, C::TILE_BYTES);
-      for (int c = 0; c < C::CHUNKS; ++c)
-        tma_load_4d(smem + C::OFF_Q + c * C::CHUNK_BYTES, &p.tm_q[role], q_full, c * 64, qt * BM, h, b);
+      int k_issued = 0, v_issued = 0;  // K / V tiles whose loads were issued
+      mbar_arrive_expect_tx(q_full, C::TILE_BYTES * (has_b ? 2 : 1));
+      for (int t = 0; t < (has_b ? 2 : 1); ++t)
+        for (int c = 0; c < C::CHUNKS; ++c)
+          tma_load_4d(smem + C::OFF_Q + t * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_q[role], q_full, c * 64,
+                      (tileA + t) * BM, h, b);
       for (int j = 0; j < nkv; ++j) {
         const int s = j % S;
         const uint32_t ph = (j / S) & 1;
@@ -179,20 +250,23 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
         for (int c = 0; c < C::CHUNKS; ++c)
           tma_load_4d(smem + C::OFF_K + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_k[r], k_full + s,
                       c * 64, row0, h, b);
-        ++k_issued[s];
+        ++k_issued;
         if (j >= S && !mbar_wait(v_empty + s, ph ^ 1, ctl)) break;
         mbar_arrive_expect_tx(v_full + s, C::TILE_BYTES);
         for (int c = 0; c < C::CHUNKS; ++c)
           tma_load_4d(smem + C::OFF_V + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_v[r], v_full + s,
                       c * 64, row0, h, b);
-        ++v_issued[s];
+        ++v_issued;
       }
       if (*abort_flag) {
-        // Let every load this thread issued land before the CTA exits.
+        // Let every load this thread issued land before the CTA exits: stage s
+        // received loads for j = s, s + S, ...; wait for the last one's phase.
         mbar_wait_drain(q_full, 0, p.budget_ns);
         for (int s = 0; s < S; ++s) {
-          if (k_issued[s] > 0) mbar_wait_drain(k_full + s, (k_issued[s] - 1) & 1, p.budget_ns);
-          if (v_issued[s] > 0) mbar_wait_drain(v_full + s, (v_issued[s] - 1) & 1, p.budget_ns);
+          const int nk = (k_issued > s) ? (k_issued - s + S - 1) / S : 0;
+          const int nv = (v_issued > s) ? (v_issued - s + S - 1) / S : 0;
+          if (nk > 0) mbar_wait_drain(k_full + s, (nk - 1) & 1, p.budget_ns);
+          if (nv > 0) mbar_wait_drain(v_full + s, (nv - 1) & 1, p.budget_ns);
         }
       }
     }
@@ -204,43 +278,51 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
       const uint32_t sq = smem_u32(smem + C::OFF_Q);
       const uint32_t sk = smem_u32(smem + C::OFF_K);
       const uint32_t sv = smem_u32(smem + C::OFF_V);
+      const int ntile = has_b ? 2 : 1;
       bool issued_any = false;
-      auto issue_qk = [&](int j) -> bool {
+      auto qk = [&](int j, int t) {
         const int s = j % S;
-        if (!mbar_wait(k_full + s, (j / S) & 1, ctl)) return false;
-        tc_fence_after();
-        const uint32_t d_t = tmem + ((j & 1) ? C::TM_S1 : C::TM_S0);
+        const uint32_t d_t = tmem + C::TM_S + 128 * t;
+        const uint32_t qbase = sq + t * C::TILE_BYTES;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
-          umma_ss(d_t, sdesc_sw128(sq + off, 16, 1024), sdesc_sw128(sk + s * C::TILE_BYTES + off, 16, 1024),
+          umma_ss(d_t, sdesc_sw128(qbase + off, 16, 1024), sdesc_sw128(sk + s * C::TILE_BYTES + off, 16, 1024),
                   IDESC_QK, kk > 0 ? 1u : 0u);
         }
-        issued_any = true;
-        umma_commit(s_full + (j & 1));
-        umma_commit(k_empty + s);
-        return true;
+        umma_commit(s_full + t);
       };
-      bool ok = mbar_wait(q_full, 0, ctl);
+      auto pv = [&](int j, int t) {
+        const int s = j % S;
+        const uint32_t p_t = tmem + C::TM_S + 128 * t;
+        const uint32_t o_t = tmem + C::TM_O + 128 * t;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk)
+          umma_ts(o_t, p_t + kk * 8, sdesc_sw128(sv + s * C::TILE_BYTES + kk * 16 * 128, C::CHUNK_BYTES, 1024),
+                  IDESC_PV, (j > 0 || kk > 0) ? 1u : 0u);
+        umma_commit(o_done + t);
+      };
+      bool ok = mbar_wait(q_full, 0, ctl) && mbar_wait(k_full, 0, ctl);
       if (ok) {
         tc_fence_after();
-        ok = issue_qk(0);
+        for (int t = 0; t < ntile; ++t) qk(0, t);
+        umma_commit(k_empty);
+        issued_any = true;
       }
       for (int j = 0; ok && j < nkv; ++j) {
-        if (j + 1 < nkv && !(ok = issue_qk(j + 1))) break;
-        if (!(ok = mbar_wait(p_ready + (j & 1), (j >> 1) & 1, ctl))) break;
         const int s = j % S;
+        const bool next = j + 1 < nkv;
         if (!(ok = mbar_wait(v_full + s, (j / S) & 1, ctl))) break;
-        tc_fence_after();
-        const uint32_t p_t = tmem + ((j & 1) ? C::TM_S1 : C::TM_S0);
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
-          umma_ts(tmem + C::TM_O, p_t + kk * 8,
-                  sdesc_sw128(sv + s * C::TILE_BYTES + kk * 16 * 128, C::CHUNK_BYTES, 1024), IDESC_PV,
-                  (j > 0 || kk > 0) ? 1u : 0u);
+        if (next && !(ok = mbar_wait(k_full + (j + 1) % S, ((j + 1) / S) & 1, ctl))) break;
+        for (int t = 0; t < ntile; ++t) {
+          if (!(ok = mbar_wait(p_ready + t, j & 1, ctl))) break;
+          tc_fence_after();
+          pv(j, t);
+          if (next) qk(j + 1, t);  // S_t is free: PV_t(j) was issued first
         }
+        if (!ok) break;
         umma_commit(v_empty + s);
-        umma_commit(o_done);
+        if (next) umma_commit(k_empty + (j + 1) % S);
       }
       if (!ok && issued_any) {
         umma_commit(drain);
@@ -249,35 +331,34 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
     }
   } else {
     // -------------------------------------------------------------- softmax
-    const int quarter = warp & 3;  // TMEM lane quarter this warp may access
+    const int t = (warp >= 6) ? 1 : 0;   // which Q tile this warpgroup owns
+    const int quarter = warp & 3;        // TMEM lane quarter this warp may access
     const int row = quarter * 32 + lane;
     const uint32_t lane_off = uint32_t(quarter * 32) << 16;
+    const uint32_t s_t = tmem + lane_off + C::TM_S + 128 * t;
+    const uint32_t o_t = tmem + lane_off + C::TM_O + 128 * t;
+    const int tile = tileA + t;
+    const bool active = (t == 0) || has_b;
     const float sl2 = p.scale_log2;
     const float bias_l2 = (role == 2 && p.bias) ? __ldg(p.bias + h) * kLog2e : 0.f;
     float m = -INFINITY, l = 0.f, lref = 0.f;
-    bool ok = true;
-    for (int j = 0; j < nkv; ++j) {
+    bool ok = active;
+    for (int j = 0; ok && j < nkv; ++j) {
       int r, row0;
       kv_tile(p, j, r, row0);
       const int nvalid = min(BN, p.n[r] - row0);
       const float badd = (r == 1) ? bias_l2 : 0.f;
-      ok = __all_sync(0xffffffffu, mbar_wait(s_full + (j & 1), (j >> 1) & 1, ctl));
+      ok = __all_sync(0xffffffffu, mbar_wait(s_full + t, j & 1, ctl));
       if (!ok) break;
       tc_fence_after();
-      const uint32_t s_t = tmem + lane_off + ((j & 1) ? C::TM_S1 : C::TM_S0);
-      uint32_t sa[32], sb[32], sc[32], sd[32];
-      tmem_ld32(s_t + 0, sa);
-      tmem_ld32(s_t + 32, sb);
-      tmem_ld32(s_t + 64, sc);
-      tmem_ld32(s_t + 96, sd);
-      tmem_ld_wait();
+      // Pass 1: row max over the tile (two 64-column TMEM reads).
+      const bool tail = nvalid < BN;
       float mx = -INFINITY;
 #pragma unroll
-      for (int c = 0; c < 32; ++c) {
-        if (c < nvalid) mx = fmaxf(mx, __uint_as_float(sa[c]));
-        if (c + 32 < nvalid) mx = fmaxf(mx, __uint_as_float(sb[c]));
-        if (c + 64 < nvalid) mx = fmaxf(mx, __uint_as_float(sc[c]));
-        if (c + 96 < nvalid) mx = fmaxf(mx, __uint_as_float(sd[c]));
+      for (int hf = 0; hf < 2; ++hf) {
+        float v[64];
+        tmem_ld64(s_t + 64 * hf, v);
+        mx = tail ? max64<true>(v, 64 * hf, nvalid, mx) : max64<false>(v, 64 * hf, nvalid, mx);
       }
       const float mt = fmaf(mx, sl2, badd);  // tile max, log2 units
       float alpha = 1.f;
@@ -289,53 +370,43 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
         lref *= alpha;
         m = mt;
       }
-      const float negm = badd - m;
+      // Pass 2: P_j over the first 64 columns of S_t (half hf of the logits ->
+      // columns [32 hf, 32 hf + 32)), never over logits still to be read. The
+      // previous P in this buffer was consumed by PV_t(j-1), which completed
+      // before QK_t(j) wrote S_t.
+      const uint64_t scale2 = f2_pack(sl2, sl2);
+      const uint64_t off2 = f2_pack(badd - m, badd - m);
       float rs = 0.f;
-      uint32_t pa[32], pb[32];
 #pragma unroll
-      for (int c = 0; c < 16; ++c) {
-        const float x0 = (2 * c < nvalid) ? ex2_approx(fmaf(__uint_as_float(sa[2 * c]), sl2, negm)) : 0.f;
-        const float x1 = (2 * c + 1 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sa[2 * c + 1]), sl2, negm)) : 0.f;
-        const float y0 = (2 * c + 32 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sb[2 * c]), sl2, negm)) : 0.f;
-        const float y1 =
-            (2 * c + 33 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sb[2 * c + 1]), sl2, negm)) : 0.f;
-        const float z0 = (2 * c + 64 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sc[2 * c]), sl2, negm)) : 0.f;
-        const float z1 =
-            (2 * c + 65 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sc[2 * c + 1]), sl2, negm)) : 0.f;
-        const float w0 = (2 * c + 96 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sd[2 * c]), sl2, negm)) : 0.f;
-        const float w1 =
-            (2 * c + 97 < nvalid) ? ex2_approx(fmaf(__uint_as_float(sd[2 * c + 1]), sl2, negm)) : 0.f;
-        rs += (x0 + x1) + (y0 + y1) + (z0 + z1) + (w0 + w1);
-        pa[c] = pack_bf16x2(x0, x1);
-        pa[c + 16] = pack_bf16x2(y0, y1);
-        pb[c] = pack_bf16x2(z0, z1);
-        pb[c + 16] = pack_bf16x2(w0, w1);
+      for (int hf = 0; hf < 2; ++hf) {
+        float v[64];
+        tmem_ld64(s_t + 64 * hf, v);
+        rs += tail ? exp64_store<true>(v, 64 * hf, nvalid, scale2, off2, s_t + 32 * hf)
+                   : exp64_store<false>(v, 64 * hf, nvalid, scale2, off2, s_t + 32 * hf);
       }
       l += rs;
       if (r == 1) lref += rs;
       if (__any_sync(0xffffffffu, resc)) {
-        ok = __all_sync(0xffffffffu, mbar_wait(o_done, (j - 1) & 1, ctl));
+        ok = __all_sync(0xffffffffu, mbar_wait(o_done + t, (j - 1) & 1, ctl));
         if (!ok) break;
         tc_fence_after();
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t ov[32];
-          tmem_ld32(tmem + lane_off + C::TM_O + c0, ov);
+          tmem_ld32(o_t + c0, ov);
           tmem_ld_wait();
 #pragma unroll
           for (int i = 0; i < 32; ++i) ov[i] = __float_as_uint(__uint_as_float(ov[i]) * alpha);
-          tmem_st32(tmem + lane_off + C::TM_O + c0, ov);
+          tmem_st32(o_t + c0, ov);
         }
       }
-      tmem_st32(s_t + 0, pa);
-      tmem_st32(s_t + 32, pb);
       tmem_st_wait();
       tc_fence_before();
-      mbar_arrive(p_ready + (j & 1));
+      mbar_arrive(p_ready + t);
     }
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done, (nkv - 1) & 1, ctl));
-    const int grow = qt * BM + row;
-    const bool valid = grow < p.n[role];
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done + t, (nkv - 1) & 1, ctl));
+    const int grow = tile * BM + row;
+    const bool valid = active && grow < p.n[role];
     const float inv_l = 1.f / l;
     if (ok) {
       tc_fence_after();
@@ -343,7 +414,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
 #pragma unroll
       for (int c0 = 0; c0 < D; c0 += 32) {
         uint32_t ov[32];
-        tmem_ld32(tmem + lane_off + C::TM_O + c0, ov);
+        tmem_ld32(o_t + c0, ov);
         tmem_ld_wait();
         uint32_t pk[16];
 #pragma unroll
@@ -364,11 +435,12 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
     float mv = (ok && valid && in_mass) ? lref * inv_l : 0.f;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mv += __shfl_xor_sync(0xffffffffu, mv, o);
-    if (lane == 0) red[quarter] = mv;
-    named_bar_sync(1, 128);
-    if (ok && role != 1 && quarter == 0 && lane == 0) {
-      const int idx = (role == 0) ? qt : p.q_tiles[0] + qt;
-      p.mass_partial[(int64_t(b) * p.H + h) * p.mpl + idx] = ((red[0] + red[1]) + red[2]) + red[3];
+    if (lane == 0) red[4 * t + quarter] = mv;
+    named_bar_sync(1 + t, 128);
+    if (ok && active && role != 1 && quarter == 0 && lane == 0) {
+      const int idx = (role == 0) ? tile : p.q_tiles[0] + tile;
+      p.mass_partial[(int64_t(b) * p.H + h) * p.mpl + idx] =
+          ((red[4 * t] + red[4 * t + 1]) + red[4 * t + 2]) + red[4 * t + 3];
     }
   }
   tc_fence_before();
@@ -511,11 +583,13 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
     p.n[r] = n;
     p.kv_tiles[r] = (n + BN - 1) / BN;
     p.q_tiles[r] = (n + BM - 1) / BM;
+    p.q_blocks[r] = (p.q_tiles[r] + 1) / 2;
     if (n == 0) continue;
     if (!encode_seg(&p.tm_k[r], a->k[r], a->B, a->H, d, BN) || !encode_seg(&p.tm_v[r], a->v[r], a->B, a->H, d, BN))
       return RA_EINVAL;
     if (r == RA_REF && !ref_rows) {
       p.q_tiles[r] = 0;
+      p.q_blocks[r] = 0;
       continue;
     }
     if (!encode_seg(&p.tm_q[r], a->q[r], a->B, a->H, d, BM)) return RA_EINVAL;
@@ -536,8 +610,8 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
   p.mass_partial = a->mass_partial;
   p.err_word = a->err_word;
   p.budget_ns = wait_budget_ns();
-  const int tiles = p.q_tiles[0] + p.q_tiles[1] + p.q_tiles[2];
-  dim3 grid(tiles, a->H, a->B);
+  const int blocks = p.q_blocks[0] + p.q_blocks[1] + p.q_blocks[2];
+  dim3 grid(blocks, a->H, a->B);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   return d == 128 ? launch<128>(p, grid, st) : launch<64>(p, grid, st);
 }

@@ -22,7 +22,7 @@ namespace qd {
 
 constexpr int THREADS = 256;
 constexpr int MAX_SPLITS = 128;
-constexpr int UNROLL = 4;
+constexpr int UNROLL = 8;
 
 struct Params {
   const __nv_bfloat16* qc;
@@ -52,32 +52,35 @@ __device__ __forceinline__ void acc16(const uint4& a, const uint4& b, float& sd,
   }
 }
 
+// Thread t always reads the same 16-byte column v = t % vec_per_row of rows
+// r0 + t / vec_per_row, stepping THREADS / vec_per_row rows at a time, so the
+// loop needs no division and a warp reads whole contiguous rows.
 __global__ void __launch_bounds__(THREADS) q_delta_kernel(const Params p) {
   const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const int bh = b * p.H + h;
   const int r0 = split * p.rows_per_split;
   const int r1 = min(p.n, r0 + p.rows_per_split);
-  const int nvec = max(0, r1 - r0) * p.vec_per_row;
-  const __nv_bfloat16* qc = p.qc + b * p.c_sb + h * p.c_sh;
-  const __nv_bfloat16* qp = p.qp + b * p.p_sb + h * p.p_sh;
+  const int vpr = p.vec_per_row;
+  const int rstep = THREADS / vpr;
+  const int v = threadIdx.x % vpr;
+  const __nv_bfloat16* qc = p.qc + b * p.c_sb + h * p.c_sh + v * 8;
+  const __nv_bfloat16* qp = p.qp + b * p.p_sb + h * p.p_sh + v * 8;
   float sd = 0.f, sp = 0.f;
-  int i = threadIdx.x;
-  for (; i + (UNROLL - 1) * THREADS < nvec; i += UNROLL * THREADS) {
+  int row = r0 + threadIdx.x / vpr;
+  for (; row + (UNROLL - 1) * rstep < r1; row += UNROLL * rstep) {
     uint4 a[UNROLL], c[UNROLL];
 #pragma unroll
     for (int u = 0; u < UNROLL; ++u) {
-      const int idx = i + u * THREADS;
-      const int row = r0 + idx / p.vec_per_row, v = idx % p.vec_per_row;
-      a[u] = __ldg(reinterpret_cast<const uint4*>(qc + row * p.c_sn) + v);
-      c[u] = __ldg(reinterpret_cast<const uint4*>(qp + row * p.p_sn) + v);
+      const int64_t rr = row + u * rstep;
+      a[u] = __ldg(reinterpret_cast<const uint4*>(qc + rr * p.c_sn));
+      c[u] = __ldg(reinterpret_cast<const uint4*>(qp + rr * p.p_sn));
     }
 #pragma unroll
     for (int u = 0; u < UNROLL; ++u) acc16(a[u], c[u], sd, sp);
   }
-  for (; i < nvec; i += THREADS) {
-    const int row = r0 + i / p.vec_per_row, v = i % p.vec_per_row;
-    const uint4 a = __ldg(reinterpret_cast<const uint4*>(qc + row * p.c_sn) + v);
-    const uint4 c = __ldg(reinterpret_cast<const uint4*>(qp + row * p.p_sn) + v);
+  for (; row < r1; row += rstep) {
+    const uint4 a = __ldg(reinterpret_cast<const uint4*>(qc + int64_t(row) * p.c_sn));
+    const uint4 c = __ldg(reinterpret_cast<const uint4*>(qp + int64_t(row) * p.p_sn));
     acc16(a, c, sd, sp);
   }
   // CTA reduction in fp64, fixed order.
@@ -109,16 +112,25 @@ __global__ void __launch_bounds__(THREADS) q_delta_kernel(const Params p) {
     last = (ticket == uint32_t(p.splits - 1));
   }
   __syncthreads();
-  if (last && threadIdx.x == 0) {
+  if (last && warp == 0) {
+    // The slab's last CTA: lane i adds splits i, i + 32, ... (L2 reads), then
+    // a butterfly finishes the sum; the order is fixed, so D is deterministic.
     __threadfence();
-    const volatile double* base = p.partial + int64_t(bh) * MAX_SPLITS * 2;
+    const double* base = p.partial + int64_t(bh) * MAX_SPLITS * 2;
     double td = 0.0, tp = 0.0;
-    for (int s = 0; s < p.splits; ++s) {
-      td += base[2 * s];
-      tp += base[2 * s + 1];
+    for (int s = lane; s < p.splits; s += 32) {
+      td += __ldcg(base + 2 * s);
+      tp += __ldcg(base + 2 * s + 1);
     }
-    p.d_out[bh] = float(sqrt(td) / (sqrt(tp) + double(p.eps)));
-    p.counter[bh] = 0u;  // re-arm for the next call
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      td += __shfl_xor_sync(0xffffffffu, td, o);
+      tp += __shfl_xor_sync(0xffffffffu, tp, o);
+    }
+    if (lane == 0) {
+      p.d_out[bh] = float(sqrt(td) / (sqrt(tp) + double(p.eps)));
+      p.counter[bh] = 0u;  // re-arm for the next call
+    }
   }
 }
 
