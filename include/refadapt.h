@@ -145,6 +145,31 @@ size_t refadapt_q_delta_workspace_size(int32_t B, int32_t H);
 ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
                            float eps, float* d_out, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ------------------------------------------------------------------ Q change, no allocation
+ * refadapt_q_delta_noalloc — the same D as refadapt_q_delta, for callers that
+ * cannot allocate device memory and have no workspace to hand over: for
+ * example a plugin inside a host framework that owns the whole device memory
+ * pool and forbids direct cudaMalloc, or a latency-critical loop that must not
+ * pay cudaMalloc's implicit device synchronisation. The paper has no
+ * counterpart; this is an interface convenience only.
+ *
+ * The scratch (ticket counters and per-block partial sums) lives in a
+ * file-scope static device array inside the library, sized for at most
+ * RA_Q_DELTA_NOALLOC_MAX_BH (= B * H) slabs, about 193 KB; every GPU that loads
+ * the library holds it until the process exits. Larger B * H returns RA_EINVAL
+ * (use refadapt_q_delta with a workspace). The call allocates nothing: no
+ * cudaMalloc, no cudaFree, no allocating library routine. Its first call on a
+ * device looks the array's device address up once (cudaGetSymbolAddress with
+ * that device current) and caches it; make that first call before any stream
+ * capture. Every call clears the counters on `stream` before its kernel; all
+ * calls share the one array, so calls that overlap on the GPU (different
+ * streams, or different host threads without ordering) race and must not be
+ * issued. Arguments and results are those of refadapt_q_delta.
+ */
+#define RA_Q_DELTA_NOALLOC_MAX_BH 96
+ra_status refadapt_q_delta_noalloc(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
+                                   float eps, float* d_out, void* stream);
+
 /* ------------------------------------------------------------------ gate
  * Controller state of Algorithm 1 for one trajectory (opaque, device
  * resident): a_full (step of the last full refresh), whether the current

@@ -14,13 +14,14 @@ RA_OK, RA_EINVAL, RA_EUNSUPPORTED, RA_ECUDA, RA_ETIMEOUT = 0, 1, 2, 3, 4
 RA_MODE_REUSE, RA_MODE_BOUNDARY, RA_MODE_COMPUTE, RA_MODE_FULL = 0, 1, 2, 3
 RA_TEXT, RA_REF, RA_TGT = 0, 1, 2
 RA_MASS_TILE_ROWS = 128
+RA_Q_DELTA_NOALLOC_MAX_BH = 96
 
 EXPORTED = (
     "refadapt_joint_attn", "refadapt_mass_partial_len", "refadapt_q_delta_workspace_size",
     "refadapt_q_delta", "refadapt_state_size", "refadapt_state_init", "refadapt_gate",
     "refadapt_ref_cache_update", "refadapt_status_string", "refadapt_last_error",
     "refadapt_set_wait_budget_ns", "refadapt_check_error", "refadapt_version",
-    "refadapt_selftest_wait_timeout",
+    "refadapt_selftest_wait_timeout", "refadapt_q_delta_noalloc",
 )
 
 
@@ -97,6 +98,9 @@ def load():
     lib.refadapt_check_error.argtypes = [c_void_p, c_void_p]
     lib.refadapt_version.restype = c_int32
     lib.refadapt_version.argtypes = []
+    lib.refadapt_q_delta_noalloc.restype = c_int32
+    lib.refadapt_q_delta_noalloc.argtypes = [POINTER(RaSeg), POINTER(RaSeg), c_int32, c_int32, c_int32, c_float,
+                                             c_void_p, c_void_p]
     lib.refadapt_selftest_wait_timeout.restype = c_int32
     lib.refadapt_selftest_wait_timeout.argtypes = [c_void_p, c_uint64, c_void_p]
     _lib = lib

@@ -13,7 +13,7 @@ from . import _lib
 from ._lib import RaAttnArgs, RaGateArgs, RaSeg, check
 
 __all__ = ["seg", "refadapt_joint_attn", "refadapt_mass_partial_len", "refadapt_q_delta",
-           "refadapt_q_delta_workspace_size", "refadapt_state_size", "refadapt_state_init",
+           "refadapt_q_delta_workspace_size", "refadapt_q_delta_noalloc", "refadapt_state_size", "refadapt_state_init",
            "refadapt_gate", "refadapt_ref_cache_update", "refadapt_set_wait_budget_ns",
            "refadapt_check_error", "refadapt_version", "refadapt_selftest_wait_timeout", "q_delta_workspace", "new_state",
            "alloc_mass_partial"]
@@ -87,6 +87,16 @@ def refadapt_q_delta(q_cur, q_prev, d_out, workspace, eps=1e-6, stream=None):
     return check("refadapt_q_delta", lib.refadapt_q_delta(
         ctypes.byref(sc), ctypes.byref(sp), B, H, d, float(eps), _ptr(d_out), _ptr(workspace),
         workspace.numel() * workspace.element_size(), _stream(stream)))
+
+
+def refadapt_q_delta_noalloc(q_cur, q_prev, d_out, eps=1e-6, stream=None):
+    """refadapt_q_delta without a workspace (static scratch inside the library;
+    B * H <= RA_Q_DELTA_NOALLOC_MAX_BH; calls must not overlap on the GPU)."""
+    lib = _lib.load()
+    B, H, _, d = q_cur.shape
+    sc, sp = seg(q_cur), seg(q_prev)
+    return check("refadapt_q_delta_noalloc", lib.refadapt_q_delta_noalloc(
+        ctypes.byref(sc), ctypes.byref(sp), B, H, d, float(eps), _ptr(d_out), _stream(stream)))
 
 
 def refadapt_state_size(B) -> int:

@@ -14,6 +14,7 @@
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <mutex>
 
 #include "api_common.h"
 
@@ -209,4 +210,68 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
   dim3 grid(splits, H, B);
   qd::q_delta_kernel<<<grid, qd::THREADS, 0, static_cast<cudaStream_t>(stream)>>>(p);
   return launch_status("refadapt_q_delta");
+}
+
+// ---------------------------------------------------------------------------
+// No-allocation variant: the workspace is a file-scope static device array.
+// Host code must not hand the array's name to a kernel (it is a host-side
+// stand-in); the device address comes from cudaGetSymbolAddress, looked up
+// once per device with that device current.
+namespace ra {
+namespace qd {
+
+constexpr int kNoAllocMaxBH = RA_Q_DELTA_NOALLOC_MAX_BH;
+constexpr size_t kNoAllocCounterBytes = ((size_t(kNoAllocMaxBH) * sizeof(uint32_t)) + 255) / 256 * 256;
+constexpr size_t kNoAllocBytes = kNoAllocCounterBytes + size_t(kNoAllocMaxBH) * MAX_SPLITS * 2 * sizeof(double);
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[64] = {nullptr};
+}  // namespace
+
+// Device address of g_noalloc_scratch on the current device (nullptr + error on failure).
+void* noalloc_scratch() {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    set_error("refadapt_q_delta_noalloc: no usable current device");
+    return nullptr;
+  }
+  std::lock_guard<std::mutex> lk(g_noalloc_mu);
+  if (g_noalloc_ptr[dev] == nullptr) {
+    void* ptr = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+    if (e != cudaSuccess || ptr == nullptr) {
+      set_error("refadapt_q_delta_noalloc: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
+      return nullptr;
+    }
+    g_noalloc_ptr[dev] = ptr;
+  }
+  return g_noalloc_ptr[dev];
+}
+
+}  // namespace qd
+}  // namespace ra
+
+extern "C" ra_status refadapt_q_delta_noalloc(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H,
+                                              int32_t d, float eps, float* d_out, void* stream) {
+  using namespace ra;
+  clear_error();
+  if (B < 1 || H < 1 || int64_t(B) * H > qd::kNoAllocMaxBH) {
+    set_error("refadapt_q_delta_noalloc: B * H = %lld outside [1, %d], the size of the static scratch; "
+              "use refadapt_q_delta with a workspace",
+              (long long)B * H, qd::kNoAllocMaxBH);
+    return RA_EINVAL;
+  }
+  void* scratch = qd::noalloc_scratch();
+  if (scratch == nullptr) return RA_ECUDA;
+  // The ticket counters must start at zero; the array keeps the last call's contents.
+  const size_t counters = ((size_t(B) * H * sizeof(uint32_t)) + 255) / 256 * 256;
+  const cudaError_t e = cudaMemsetAsync(scratch, 0, counters, static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    set_error("refadapt_q_delta_noalloc: cudaMemsetAsync: %s", cudaGetErrorString(e));
+    return RA_ECUDA;
+  }
+  return refadapt_q_delta(q_cur, q_prev, B, H, d, eps, d_out, scratch, qd::kNoAllocBytes, stream);
 }
