@@ -1,6 +1,7 @@
 // Host-side helpers shared by the C-ABI entry points: argument checks, the
 // thread-local error message, device properties and the wait budget.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstdint>
@@ -19,6 +20,11 @@ int num_sms();  // of the current device (cached per device)
 // A bf16 segment usable by 16-byte vector access and by TMA: 16-byte aligned
 // pointer and strides, n >= 0, non-negative strides. `what` names it in errors.
 bool check_seg(const ra_seg& s, const char* what, bool allow_null_if_empty = true);
+
+// 4-D TMA tensor map (c, n, head, sample) over one bf16 segment of head dim d,
+// box box_cols x box_rows, 128-byte swizzle or none, zero fill out of bounds.
+bool encode_seg(CUtensorMap* tm, const ra_seg& s, int B, int H, int d, int box_cols, int box_rows,
+                bool swizzle128);
 
 inline ra_status launch_status(const char* what) {
   cudaError_t e = cudaGetLastError();

@@ -1,4 +1,6 @@
 // Status strings, error message, wait budget and the error-word check.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <atomic>
@@ -61,6 +63,52 @@ bool check_seg(const ra_seg& s, const char* what, bool allow_null_if_empty) {
   }
   if (s.stride_b % 8 || s.stride_h % 8 || s.stride_n % 8) {
     set_error("%s: strides must be multiples of 8 elements (16 bytes)", what);
+    return false;
+  }
+  return true;
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
+  });
+  return fn;
+}
+
+bool encode_seg(CUtensorMap* tm, const ra_seg& s, int B, int H, int d, int box_cols, int box_rows,
+                bool swizzle128) {
+  auto fn = encode_fn();
+  if (!fn) {
+    set_error("cuTensorMapEncodeTiled unavailable from the driver");
+    return false;
+  }
+  const int64_t row_bytes = int64_t(s.stride_n) * 2;
+  int64_t sh = int64_t(s.stride_h) * 2, sb = int64_t(s.stride_b) * 2;
+  // A stride of a size-1 dimension is never used; give TMA a legal one.
+  if (H == 1 && sh == 0) sh = row_bytes * (s.n > 0 ? s.n : 1);
+  if (B == 1 && sb == 0) sb = sh * H;
+  if (row_bytes == 0 && s.n > 1) {
+    set_error("segment row stride is 0");
+    return false;
+  }
+  cuuint64_t dims[4] = {cuuint64_t(d), cuuint64_t(s.n), cuuint64_t(H), cuuint64_t(B)};
+  cuuint64_t strides[3] = {cuuint64_t(row_bytes > 0 ? row_bytes : 16 * ((d * 2 + 15) / 16)), cuuint64_t(sh),
+                           cuuint64_t(sb)};
+  cuuint32_t box[4] = {cuuint32_t(box_cols), cuuint32_t(box_rows), 1u, 1u};
+  cuuint32_t es[4] = {1u, 1u, 1u, 1u};
+  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, s.ptr, dims, strides, box, es,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE,
+                  swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) {
+    set_error("cuTensorMapEncodeTiled failed (%d)", int(r));
     return false;
   }
   return true;

@@ -26,7 +26,6 @@
 // drains its own TMA and MMA work, frees TMEM, flags the caller's error word
 // and returns.
 #include <cuda.h>
-#include <cudaTypedefs.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -131,32 +130,37 @@ __device__ __forceinline__ void tmem_ld64(uint32_t taddr, float (&v)[64]) {
 }
 
 // Probabilities of 64 logits (columns col0 ..), p = 2^(v * sl2 + negm), packed
-// to bf16 into 32 TMEM columns at p_taddr. Returns their fp32 sum. TAIL masks
-// columns >= nvalid to probability 0.
+// to bf16 into 32 TMEM columns at p_taddr (16 at a time, so at most 16 packed
+// words are live). Returns their fp32 sum. TAIL masks columns >= nvalid to
+// probability 0.
 template <bool TAIL>
 __device__ __forceinline__ float exp64_store(const float (&v)[64], int col0, int nvalid, uint64_t scale2,
                                              uint64_t off2, uint32_t p_taddr) {
   uint64_t acc0 = f2_pack(0.f, 0.f), acc1 = acc0;
-  uint32_t pk[32];
 #pragma unroll
-  for (int c = 0; c < 64; c += 4) {
-    float a0, a1, b0, b1;
-    f2_unpack(f2_fma(f2_pack(v[c], v[c + 1]), scale2, off2), a0, a1);
-    f2_unpack(f2_fma(f2_pack(v[c + 2], v[c + 3]), scale2, off2), b0, b1);
-    float p0 = ex2_approx(a0), p1 = ex2_approx(a1), p2 = ex2_approx(b0), p3 = ex2_approx(b1);
-    if (TAIL) {
-      const int e = col0 + c;
-      p0 = (e < nvalid) ? p0 : 0.f;
-      p1 = (e + 1 < nvalid) ? p1 : 0.f;
-      p2 = (e + 2 < nvalid) ? p2 : 0.f;
-      p3 = (e + 3 < nvalid) ? p3 : 0.f;
+  for (int q = 0; q < 2; ++q) {
+    uint32_t pk[16];
+#pragma unroll
+    for (int c = 0; c < 32; c += 4) {
+      const int e = 32 * q + c;
+      float a0, a1, b0, b1;
+      f2_unpack(f2_fma(f2_pack(v[e], v[e + 1]), scale2, off2), a0, a1);
+      f2_unpack(f2_fma(f2_pack(v[e + 2], v[e + 3]), scale2, off2), b0, b1);
+      float p0 = ex2_approx(a0), p1 = ex2_approx(a1), p2 = ex2_approx(b0), p3 = ex2_approx(b1);
+      if (TAIL) {
+        const int g = col0 + e;
+        p0 = (g < nvalid) ? p0 : 0.f;
+        p1 = (g + 1 < nvalid) ? p1 : 0.f;
+        p2 = (g + 2 < nvalid) ? p2 : 0.f;
+        p3 = (g + 3 < nvalid) ? p3 : 0.f;
+      }
+      acc0 = f2_add(acc0, f2_pack(p0, p1));
+      acc1 = f2_add(acc1, f2_pack(p2, p3));
+      pk[c / 2] = pack_bf16x2(p0, p1);
+      pk[c / 2 + 1] = pack_bf16x2(p2, p3);
     }
-    acc0 = f2_add(acc0, f2_pack(p0, p1));
-    acc1 = f2_add(acc1, f2_pack(p2, p3));
-    pk[c / 2] = pack_bf16x2(p0, p1);
-    pk[c / 2 + 1] = pack_bf16x2(p2, p3);
+    tmem_st16(p_taddr + 16 * q, pk);
   }
-  tmem_st32(p_taddr, pk);
   float s0, s1, s2, s3;
   f2_unpack(acc0, s0, s1);
   f2_unpack(acc1, s2, s3);
@@ -351,38 +355,64 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
       ok = __all_sync(0xffffffffu, mbar_wait(s_full + t, j & 1, ctl));
       if (!ok) break;
       tc_fence_after();
-      // Pass 1: row max over the tile (two 64-column TMEM reads).
-      const bool tail = nvalid < BN;
-      float mx = -INFINITY;
-#pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        float v[64];
-        tmem_ld64(s_t + 64 * hf, v);
-        mx = tail ? max64<true>(v, 64 * hf, nvalid, mx) : max64<false>(v, 64 * hf, nvalid, mx);
-      }
-      const float mt = fmaf(mx, sl2, badd);  // tile max, log2 units
+      // The previous P in S_t was consumed by PV_t(j-1), which completed before
+      // QK_t(j) wrote S_t. The running max m only moves when the tile's max
+      // exceeds it by more than 2^8 (then O, l, l_ref are rescaled by alpha).
       float alpha = 1.f;
       bool resc = false;
-      if (mt > m + kRescaleThresh) {
-        alpha = ex2_approx(m - mt);  // 0 when m = -inf
-        resc = (j > 0);
-        l *= alpha;
-        lref *= alpha;
-        m = mt;
-      }
-      // Pass 2: P_j over the first 64 columns of S_t (half hf of the logits ->
-      // columns [32 hf, 32 hf + 32)), never over logits still to be read. The
-      // previous P in this buffer was consumed by PV_t(j-1), which completed
-      // before QK_t(j) wrote S_t.
-      const uint64_t scale2 = f2_pack(sl2, sl2);
-      const uint64_t off2 = f2_pack(badd - m, badd - m);
-      float rs = 0.f;
+      const bool tail = nvalid < BN;
+      float rs;
+      if (!tail) {
+        // Full key tile: one TMEM read of the row with the hardware row max
+        // (tcgen05.ld.red), probabilities straight from registers.
+        float va[64], vb[64];
+        float m0, m1, m2, m3;
+        tmem_ldred32_max(s_t + 0, *reinterpret_cast<uint32_t(*)[32]>(&va[0]), m0);
+        tmem_ldred32_max(s_t + 32, *reinterpret_cast<uint32_t(*)[32]>(&va[32]), m1);
+        tmem_ldred32_max(s_t + 64, *reinterpret_cast<uint32_t(*)[32]>(&vb[0]), m2);
+        tmem_ldred32_max(s_t + 96, *reinterpret_cast<uint32_t(*)[32]>(&vb[32]), m3);
+        tmem_ld_wait();
+        const float mt = fmaf(fmaxf(fmaxf(m0, m1), fmaxf(m2, m3)), sl2, badd);  // tile max, log2 units
+        if (mt > m + kRescaleThresh) {
+          alpha = ex2_approx(m - mt);  // 0 when m = -inf
+          resc = (j > 0);
+          l *= alpha;
+          lref *= alpha;
+          m = mt;
+        }
+        // P_j over the first 64 columns of S_t: the logits are all in registers.
+        const uint64_t scale2 = f2_pack(sl2, sl2);
+        const uint64_t off2 = f2_pack(badd - m, badd - m);
+        rs = exp64_store<false>(va, 0, BN, scale2, off2, s_t + 0);
+        rs += exp64_store<false>(vb, 64, BN, scale2, off2, s_t + 32);
+      } else {
+        // Tail key tile: pass 1 takes the max over the valid columns only,
+        // pass 2 re-reads the logits (half hf -> P columns [32 hf, 32 hf + 32),
+        // never over logits still to be read).
+        float mx = -INFINITY;
 #pragma unroll
-      for (int hf = 0; hf < 2; ++hf) {
-        float v[64];
-        tmem_ld64(s_t + 64 * hf, v);
-        rs += tail ? exp64_store<true>(v, 64 * hf, nvalid, scale2, off2, s_t + 32 * hf)
-                   : exp64_store<false>(v, 64 * hf, nvalid, scale2, off2, s_t + 32 * hf);
+        for (int hf = 0; hf < 2; ++hf) {
+          float v[64];
+          tmem_ld64(s_t + 64 * hf, v);
+          mx = max64<true>(v, 64 * hf, nvalid, mx);
+        }
+        const float mt = fmaf(mx, sl2, badd);
+        if (mt > m + kRescaleThresh) {
+          alpha = ex2_approx(m - mt);
+          resc = (j > 0);
+          l *= alpha;
+          lref *= alpha;
+          m = mt;
+        }
+        const uint64_t scale2 = f2_pack(sl2, sl2);
+        const uint64_t off2 = f2_pack(badd - m, badd - m);
+        rs = 0.f;
+#pragma unroll
+        for (int hf = 0; hf < 2; ++hf) {
+          float v[64];
+          tmem_ld64(s_t + 64 * hf, v);
+          rs += exp64_store<true>(v, 64 * hf, nvalid, scale2, off2, s_t + 32 * hf);
+        }
       }
       l += rs;
       if (r == 1) lref += rs;
@@ -452,51 +482,6 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
 }
 
 // ------------------------------------------------------------------ host side
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
-  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-  static std::once_flag once;
-  std::call_once(once, [] {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult q;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
-            cudaSuccess &&
-        q == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(ptr);
-  });
-  return fn;
-}
-
-// 4-D map (d, n, head, sample) over one bf16 segment, box 64 x box_rows, 128-byte swizzle.
-bool encode_seg(CUtensorMap* tm, const ra_seg& s, int B, int H, int d, int box_rows) {
-  auto fn = encode_fn();
-  if (!fn) {
-    set_error("cuTensorMapEncodeTiled unavailable from the driver");
-    return false;
-  }
-  const int64_t row_bytes = int64_t(s.stride_n) * 2;
-  int64_t sh = int64_t(s.stride_h) * 2, sb = int64_t(s.stride_b) * 2;
-  // A stride of a size-1 dimension is never used; give TMA a legal one.
-  if (H == 1 && sh == 0) sh = row_bytes * (s.n > 0 ? s.n : 1);
-  if (B == 1 && sb == 0) sb = sh * H;
-  if (row_bytes == 0 && s.n > 1) {
-    set_error("segment row stride is 0");
-    return false;
-  }
-  cuuint64_t dims[4] = {cuuint64_t(d), cuuint64_t(s.n), cuuint64_t(H), cuuint64_t(B)};
-  cuuint64_t strides[3] = {cuuint64_t(row_bytes > 0 ? row_bytes : 16 * ((d * 2 + 15) / 16)), cuuint64_t(sh),
-                           cuuint64_t(sb)};
-  cuuint32_t box[4] = {64u, cuuint32_t(box_rows), 1u, 1u};
-  cuuint32_t es[4] = {1u, 1u, 1u, 1u};
-  CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, s.ptr, dims, strides, box, es,
-                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-  if (r != CUDA_SUCCESS) {
-    set_error("cuTensorMapEncodeTiled failed (%d)", int(r));
-    return false;
-  }
-  return true;
-}
-
 template <int D>
 ra_status launch(const Params& p, dim3 grid, cudaStream_t st) {
   static std::once_flag once;
@@ -585,14 +570,14 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
     p.q_tiles[r] = (n + BM - 1) / BM;
     p.q_blocks[r] = (p.q_tiles[r] + 1) / 2;
     if (n == 0) continue;
-    if (!encode_seg(&p.tm_k[r], a->k[r], a->B, a->H, d, BN) || !encode_seg(&p.tm_v[r], a->v[r], a->B, a->H, d, BN))
+    if (!encode_seg(&p.tm_k[r], a->k[r], a->B, a->H, d, 64, BN, true) || !encode_seg(&p.tm_v[r], a->v[r], a->B, a->H, d, 64, BN, true))
       return RA_EINVAL;
     if (r == RA_REF && !ref_rows) {
       p.q_tiles[r] = 0;
       p.q_blocks[r] = 0;
       continue;
     }
-    if (!encode_seg(&p.tm_q[r], a->q[r], a->B, a->H, d, BM)) return RA_EINVAL;
+    if (!encode_seg(&p.tm_q[r], a->q[r], a->B, a->H, d, 64, BM, true)) return RA_EINVAL;
     p.o_ptr[r] = static_cast<__nv_bfloat16*>(a->o[r].ptr);
     p.o_sb[r] = a->o[r].stride_b;
     p.o_sh[r] = a->o[r].stride_h;

@@ -1,136 +1,226 @@
 // refadapt_q_delta: relative L2 change of the target query per (sample, head),
 // D = ||q_t - q_{t-1}||_F / (||q_{t-1}||_F + eps)   (paper Eq. 1, Sec. 4).
 //
-// HBM-bound: each (sample, head) slab of n rows x d columns is split into
-// `splits` row ranges, one CTA each, sized so the grid covers every SM several
-// times. A CTA streams both tensors with 16-byte loads (several in flight per
-// thread), accumulates sum (q_t - q_{t-1})^2 and sum q_{t-1}^2 in fp32 per
-// thread, reduces them in fp64 across the CTA in a fixed order and stores the
-// pair in the workspace. The last CTA of a slab to finish (ticket counter in
-// the workspace) adds the pairs in split order and writes D, then re-arms the
-// counter, so results are deterministic and the workspace is ready for the
-// next call.
+// HBM-bound streaming reduction, one CTA per SM. Work is cut into units of
+// 12 KB per tensor (48 rows at d = 128, 96 rows at d = 64) of one (sample,
+// head) slab; CTA c takes the contiguous unit range [c U / G, (c+1) U / G) in
+// slab-major order. A producer thread streams both tensors' units through an
+// 8-stage shared-memory ring, so each SM keeps up to 192 KB in flight without
+// register limits. When both tensors' rows are contiguous within a slab
+// (stride_n == d) a unit is one 1-D bulk copy of its bytes (the slab's last
+// unit is shorter); otherwise it is a 2-D TMA tensor load (any row strides;
+// rows past the slab end arrive as zeros and add nothing). Unit i goes to stage i % 8 and is
+// consumed by warp i % 8, so every stage has one consumer that waits its
+// phases in order: packed fp32 sums of (q_t - q_{t-1})^2 and q_{t-1}^2 per
+// lane, then an fp64 butterfly per unit. The CTA then adds its unit sums per
+// slab in unit order and stores one slot per (slab, CTA); the slab's last
+// contributor (ticket counter) adds the slots in CTA order and writes D, then
+// re-arms the counter. Every sum has a fixed order, so D is deterministic.
+#include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include <cmath>
+#include <cstring>
 #include <mutex>
 
 #include "api_common.h"
+#include "tc_ptx.cuh"
 
 namespace ra {
 namespace qd {
 
-constexpr int THREADS = 256;
-constexpr int MAX_SPLITS = 128;
-constexpr int UNROLL = 8;
+constexpr int MAX_SPLITS = 128;       // slots per slab in the workspace
+constexpr int CONSUMER_WARPS = 8;
+constexpr int STAGES = CONSUMER_WARPS;  // stage s belongs to consumer warp s
+constexpr int UNIT_BYTES = 12288;       // per tensor: 48 rows at d = 128, 96 at d = 64
+constexpr int THREADS = 32 * (CONSUMER_WARPS + 1);
+constexpr int MAX_UNITS_PER_CTA = 1024;
+constexpr int OFF_BAR = STAGES * 2 * UNIT_BYTES;
+constexpr int OFF_MISC = OFF_BAR + 2 * STAGES * 8;           // abort flag
+constexpr int OFF_SUMS = OFF_MISC + 16;                       // double2 per unit
+constexpr int SMEM_BYTES = OFF_SUMS + MAX_UNITS_PER_CTA * 16;
+constexpr int SMEM_ALLOC = SMEM_BYTES + 1024;
+static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 
 struct Params {
-  const __nv_bfloat16* qc;
-  const __nv_bfloat16* qp;
-  int64_t c_sb, c_sh, c_sn;
-  int64_t p_sb, p_sh, p_sn;
-  int32_t H, n, vec_per_row;  // vec = 8 bf16 = 16 bytes
-  int32_t splits, rows_per_split;
+  CUtensorMap tm_c, tm_p;  // (d, n, H, B), box (d, rows_per_unit), no swizzle
+  const char* base_c;      // 1-D bulk path: slab (b, h) starts at base + b * sb + h * sh
+  const char* base_p;
+  int64_t c_sb, c_sh, p_sb, p_sh;  // bytes
+  int64_t slab_bytes;      // n * d * 2
+  int32_t bulk;            // 1: 1-D bulk copies, 0: 2-D tensor loads
+  int32_t H, rows_per_unit;
+  int32_t per_slab;        // units per slab
+  int32_t units;           // all units
+  int32_t grid;
   float eps;
   float* d_out;
-  double* partial;     // [B*H][MAX_SPLITS][2]
-  uint32_t* counter;   // [B*H]
+  double* partial;         // [B*H][MAX_SPLITS][2]
+  uint32_t* counter;       // [B*H]
+  uint64_t budget_ns;
 };
 
-__device__ __forceinline__ void acc16(const uint4& a, const uint4& b, float& sd, float& sp) {
-  const __nv_bfloat162* x = reinterpret_cast<const __nv_bfloat162*>(&a);
-  const __nv_bfloat162* y = reinterpret_cast<const __nv_bfloat162*>(&b);
+// CTA that owns unit u under the balanced split of U units over G CTAs.
+__device__ __forceinline__ int owner(int64_t u, int64_t U, int64_t G) {
+  return int(((u + 1) * G + U - 1) / U - 1);
+}
+
+// Sums over one 16-byte vector pair: (c - p)^2 and p^2, two lanes of fp32 at a time.
+__device__ __forceinline__ void acc16(const uint4& c, const uint4& p, uint64_t& sd, uint64_t& sp) {
+  const uint32_t cw[4] = {c.x, c.y, c.z, c.w};
+  const uint32_t pw[4] = {p.x, p.y, p.z, p.w};
+  const uint64_t neg1 = f2_pack(-1.f, -1.f);
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const float2 fx = __bfloat1622float2(x[i]);
-    const float2 fy = __bfloat1622float2(y[i]);
-    const float d0 = fx.x - fy.x, d1 = fx.y - fy.y;
-    sd = fmaf(d0, d0, sd);
-    sd = fmaf(d1, d1, sd);
-    sp = fmaf(fy.x, fy.x, sp);
-    sp = fmaf(fy.y, fy.y, sp);
+    const uint64_t cc = f2_pack(__uint_as_float(cw[i] << 16), __uint_as_float(cw[i] & 0xFFFF0000u));
+    const uint64_t pp = f2_pack(__uint_as_float(pw[i] << 16), __uint_as_float(pw[i] & 0xFFFF0000u));
+    const uint64_t df = f2_fma(pp, neg1, cc);  // exact: both are bf16 values
+    sd = f2_fma(df, df, sd);
+    sp = f2_fma(pp, pp, sp);
   }
 }
 
-// Thread t always reads the same 16-byte column v = t % vec_per_row of rows
-// r0 + t / vec_per_row, stepping THREADS / vec_per_row rows at a time, so the
-// loop needs no division and a warp reads whole contiguous rows.
-__global__ void __launch_bounds__(THREADS) q_delta_kernel(const Params p) {
-  const int split = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
-  const int bh = b * p.H + h;
-  const int r0 = split * p.rows_per_split;
-  const int r1 = min(p.n, r0 + p.rows_per_split);
-  const int vpr = p.vec_per_row;
-  const int rstep = THREADS / vpr;
-  const int v = threadIdx.x % vpr;
-  const __nv_bfloat16* qc = p.qc + b * p.c_sb + h * p.c_sh + v * 8;
-  const __nv_bfloat16* qp = p.qp + b * p.p_sb + h * p.p_sh + v * 8;
-  float sd = 0.f, sp = 0.f;
-  int row = r0 + threadIdx.x / vpr;
-  for (; row + (UNROLL - 1) * rstep < r1; row += UNROLL * rstep) {
-    uint4 a[UNROLL], c[UNROLL];
-#pragma unroll
-    for (int u = 0; u < UNROLL; ++u) {
-      const int64_t rr = row + u * rstep;
-      a[u] = __ldg(reinterpret_cast<const uint4*>(qc + rr * p.c_sn));
-      c[u] = __ldg(reinterpret_cast<const uint4*>(qp + rr * p.p_sn));
-    }
-#pragma unroll
-    for (int u = 0; u < UNROLL; ++u) acc16(a[u], c[u], sd, sp);
-  }
-  for (; row < r1; row += rstep) {
-    const uint4 a = __ldg(reinterpret_cast<const uint4*>(qc + int64_t(row) * p.c_sn));
-    const uint4 c = __ldg(reinterpret_cast<const uint4*>(qp + int64_t(row) * p.p_sn));
-    acc16(a, c, sd, sp);
-  }
-  // CTA reduction in fp64, fixed order.
-  double dd = sd, dp = sp;
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) {
-    dd += __shfl_xor_sync(0xffffffffu, dd, o);
-    dp += __shfl_xor_sync(0xffffffffu, dp, o);
-  }
-  __shared__ double red[2][THREADS / 32];
-  __shared__ bool last;
+__global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_constant__ Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
+  uint64_t* empty = full + STAGES;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + OFF_MISC);
+  double* sums = reinterpret_cast<double*>(smem + OFF_SUMS);
+  const int c = blockIdx.x;
+  const int u0 = int(int64_t(c) * p.units / p.grid);
+  const int u1 = int(int64_t(c + 1) * p.units / p.grid);
+  const int nu = u1 - u0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (lane == 0) {
-    red[0][warp] = dd;
-    red[1][warp] = dp;
-  }
-  __syncthreads();
   if (threadIdx.x == 0) {
-    double td = 0.0, tp = 0.0;
-    for (int w = 0; w < THREADS / 32; ++w) {
-      td += red[0][w];
-      tp += red[1][w];
+    for (int s = 0; s < STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
     }
-    double* slot = p.partial + (int64_t(bh) * MAX_SPLITS + split) * 2;
-    slot[0] = td;
-    slot[1] = tp;
-    __threadfence();
-    const uint32_t ticket = atomicAdd(p.counter + bh, 1u);
-    last = (ticket == uint32_t(p.splits - 1));
+    *abort_flag = 0;
+    fence_mbar_init();
   }
   __syncthreads();
-  if (last && warp == 0) {
-    // The slab's last CTA: lane i adds splits i, i + 32, ... (L2 reads), then
-    // a butterfly finishes the sum; the order is fixed, so D is deterministic.
-    __threadfence();
-    const double* base = p.partial + int64_t(bh) * MAX_SPLITS * 2;
-    double td = 0.0, tp = 0.0;
-    for (int s = lane; s < p.splits; s += 32) {
-      td += __ldcg(base + 2 * s);
-      tp += __ldcg(base + 2 * s + 1);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      td += __shfl_xor_sync(0xffffffffu, td, o);
-      tp += __shfl_xor_sync(0xffffffffu, tp, o);
-    }
+  const WaitCtl ctl{abort_flag, nullptr, p.budget_ns};
+
+  if (warp == CONSUMER_WARPS) {
     if (lane == 0) {
-      p.d_out[bh] = float(sqrt(td) / (sqrt(tp) + double(p.eps)));
-      p.counter[bh] = 0u;  // re-arm for the next call
+      // ---------------------------------------------------------- producer
+      if (!p.bulk) {
+        tma_prefetch_desc(&p.tm_c);
+        tma_prefetch_desc(&p.tm_p);
+      }
+      int issued = 0;
+      for (int i = 0; i < nu; ++i) {
+        const int s = i % STAGES;
+        if (i >= STAGES && !mbar_wait(empty + s, ((i / STAGES) - 1) & 1, ctl)) break;
+        const int u = u0 + i;
+        const int slab = u / p.per_slab, k = u % p.per_slab;
+        const int b = slab / p.H, h = slab % p.H;
+        if (p.bulk) {
+          const int64_t off = int64_t(k) * UNIT_BYTES;
+          const int64_t rem = p.slab_bytes - off;
+          const uint32_t bytes = uint32_t(rem < UNIT_BYTES ? rem : UNIT_BYTES);
+          mbar_arrive_expect_tx(full + s, 2 * bytes);
+          bulk_load(smem + s * 2 * UNIT_BYTES, p.base_c + b * p.c_sb + h * p.c_sh + off, bytes, full + s);
+          bulk_load(smem + s * 2 * UNIT_BYTES + UNIT_BYTES, p.base_p + b * p.p_sb + h * p.p_sh + off, bytes,
+                    full + s);
+        } else {
+          mbar_arrive_expect_tx(full + s, 2 * UNIT_BYTES);
+          tma_load_4d(smem + s * 2 * UNIT_BYTES, &p.tm_c, full + s, 0, k * p.rows_per_unit, h, b);
+          tma_load_4d(smem + s * 2 * UNIT_BYTES + UNIT_BYTES, &p.tm_p, full + s, 0, k * p.rows_per_unit, h, b);
+        }
+        ++issued;
+      }
+      if (*abort_flag) {
+        for (int s = 0; s < STAGES; ++s) {
+          const int n_s = (issued > s) ? (issued - s + STAGES - 1) / STAGES : 0;
+          if (n_s > 0) mbar_wait_drain(full + s, (n_s - 1) & 1, p.budget_ns);
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    for (int i = warp; i < nu; i += CONSUMER_WARPS) {
+      const int s = i % STAGES;
+      if (!__all_sync(0xffffffffu, mbar_wait(full + s, (i / STAGES) & 1, ctl))) break;
+      const uint4* vc = reinterpret_cast<const uint4*>(smem + s * 2 * UNIT_BYTES);
+      const uint4* vp = reinterpret_cast<const uint4*>(smem + s * 2 * UNIT_BYTES + UNIT_BYTES);
+      uint64_t sd = f2_pack(0.f, 0.f), sp = sd;
+      int nvec = UNIT_BYTES / 16;  // a short last unit of the bulk path holds fewer bytes
+      if (p.bulk) {
+        const int64_t rem = p.slab_bytes - int64_t((u0 + i) % p.per_slab) * UNIT_BYTES;
+        if (rem < UNIT_BYTES) nvec = int(rem / 16);
+      }
+      if (nvec == UNIT_BYTES / 16) {
+#pragma unroll 8
+        for (int m = 0; m < UNIT_BYTES / 16 / 32; ++m) acc16(vc[lane + 32 * m], vp[lane + 32 * m], sd, sp);
+      } else {
+        for (int v = lane; v < nvec; v += 32) acc16(vc[v], vp[v], sd, sp);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty + s);
+      float a0, a1, b0, b1;
+      f2_unpack(sd, a0, a1);
+      f2_unpack(sp, b0, b1);
+      double dd = double(a0) + double(a1), dp = double(b0) + double(b1);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        dd += __shfl_xor_sync(0xffffffffu, dd, o);
+        dp += __shfl_xor_sync(0xffffffffu, dp, o);
+      }
+      if (lane == 0) {
+        sums[2 * i] = dd;
+        sums[2 * i + 1] = dp;
+      }
+    }
+    named_bar_sync(1, 32 * CONSUMER_WARPS);
+    if (warp == 0) {
+      // Per slab touched by this CTA: add its unit sums in unit order, store the
+      // slot, take a ticket; the slab's last contributor finishes D.
+      const bool aborted = *abort_flag != 0;
+      int i = 0;
+      while (i < nu) {
+        const int slab = (u0 + i) / p.per_slab;
+        double td = 0.0, tp = 0.0;
+        int j = i;
+        for (; j < nu && (u0 + j) / p.per_slab == slab; ++j) {
+          td += sums[2 * j];
+          tp += sums[2 * j + 1];
+        }
+        const int64_t first_u = int64_t(slab) * p.per_slab;
+        const int64_t last_u = first_u + p.per_slab - 1;
+        const int c_lo = owner(first_u, p.units, p.grid);
+        const int count = owner(last_u, p.units, p.grid) - c_lo + 1;
+        double* slots = p.partial + int64_t(slab) * MAX_SPLITS * 2;
+        uint32_t last = 0;
+        if (lane == 0) {
+          slots[2 * (c - c_lo)] = aborted ? NAN : td;
+          slots[2 * (c - c_lo) + 1] = tp;
+          __threadfence();
+          last = (atomicAdd(p.counter + slab, 1u) == uint32_t(count - 1)) ? 1u : 0u;
+        }
+        last = __shfl_sync(0xffffffffu, last, 0);
+        if (last) {
+          __threadfence();
+          double sd = 0.0, sp = 0.0;
+          for (int q = lane; q < count; q += 32) {
+            sd += __ldcg(slots + 2 * q);
+            sp += __ldcg(slots + 2 * q + 1);
+          }
+#pragma unroll
+          for (int o = 16; o > 0; o >>= 1) {
+            sd += __shfl_xor_sync(0xffffffffu, sd, o);
+            sp += __shfl_xor_sync(0xffffffffu, sp, o);
+          }
+          if (lane == 0) {
+            p.d_out[slab] = float(sqrt(sd) / (sqrt(sp) + double(p.eps)));
+            p.counter[slab] = 0u;  // re-arm for the next call
+          }
+        }
+        i = j;
+      }
     }
   }
 }
@@ -179,36 +269,60 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
   }
   const int n = q_cur->n;
   const int bh = B * H;
-  // Enough CTAs to cover every SM about four times, at least 8 rows each.
-  const int want = (4 * num_sms() + bh - 1) / bh;
-  int splits = want < 1 ? 1 : want;
-  if (splits > qd::MAX_SPLITS) splits = qd::MAX_SPLITS;
-  const int max_by_rows = (n + 7) / 8;
-  if (splits > max_by_rows) splits = max_by_rows;
-  const int rps = (n + splits - 1) / splits;
-  splits = (n + rps - 1) / rps;
-
   qd::Params p;
-  p.qc = static_cast<const __nv_bfloat16*>(q_cur->ptr);
-  p.qp = static_cast<const __nv_bfloat16*>(q_prev->ptr);
-  p.c_sb = q_cur->stride_b;
-  p.c_sh = q_cur->stride_h;
-  p.c_sn = q_cur->stride_n;
-  p.p_sb = q_prev->stride_b;
-  p.p_sh = q_prev->stride_h;
-  p.p_sn = q_prev->stride_n;
   p.H = H;
-  p.n = n;
-  p.vec_per_row = d / 8;
-  p.splits = splits;
-  p.rows_per_split = rps;
+  p.rows_per_unit = qd::UNIT_BYTES / (2 * d);
+  p.per_slab = (n + p.rows_per_unit - 1) / p.rows_per_unit;
+  const int64_t units = int64_t(bh) * p.per_slab;
+  if (units > (int64_t(1) << 30)) {
+    set_error("refadapt_q_delta: problem too large");
+    return RA_EINVAL;
+  }
+  p.units = int(units);
+  // One CTA per SM; at most MAX_SPLITS - 1 CTAs may share a slab (slots) and
+  // at most MAX_UNITS_PER_CTA units may fall to one CTA.
+  int64_t G = num_sms();
+  if (G > units) G = units;
+  if (G > int64_t(qd::MAX_SPLITS - 1) * bh) G = int64_t(qd::MAX_SPLITS - 1) * bh;
+  while ((units + G - 1) / G > qd::MAX_UNITS_PER_CTA) G *= 2;
+  if (G > units) G = units;
+  if (G > int64_t(qd::MAX_SPLITS - 1) * bh || G > 2147483647) {
+    set_error("refadapt_q_delta: n = %d rows per slab is too large", n);
+    return RA_EINVAL;
+  }
+  p.grid = int(G);
   p.eps = eps;
   p.d_out = d_out;
   const size_t counters = ((size_t(bh) * sizeof(uint32_t)) + 255) / 256 * 256;
   p.counter = static_cast<uint32_t*>(workspace);
   p.partial = reinterpret_cast<double*>(static_cast<char*>(workspace) + counters);
-  dim3 grid(splits, H, B);
-  qd::q_delta_kernel<<<grid, qd::THREADS, 0, static_cast<cudaStream_t>(stream)>>>(p);
+  p.budget_ns = wait_budget_ns();
+  p.bulk = (q_cur->stride_n == d && q_prev->stride_n == d) ? 1 : 0;
+  p.base_c = static_cast<const char*>(q_cur->ptr);
+  p.base_p = static_cast<const char*>(q_prev->ptr);
+  p.c_sb = q_cur->stride_b * 2;
+  p.c_sh = q_cur->stride_h * 2;
+  p.p_sb = q_prev->stride_b * 2;
+  p.p_sh = q_prev->stride_h * 2;
+  p.slab_bytes = int64_t(n) * d * 2;
+  if (p.bulk) {
+    // Units are byte ranges of a slab; rows_per_unit * d * 2 == UNIT_BYTES either way.
+    std::memset(&p.tm_c, 0, sizeof(p.tm_c));
+    std::memset(&p.tm_p, 0, sizeof(p.tm_p));
+  } else if (!encode_seg(&p.tm_c, *q_cur, B, H, d, d, p.rows_per_unit, false) ||
+             !encode_seg(&p.tm_p, *q_prev, B, H, d, d, p.rows_per_unit, false)) {
+    return RA_EINVAL;
+  }
+  static std::once_flag once;
+  static cudaError_t attr_err = cudaSuccess;
+  std::call_once(once, [] {
+    attr_err = cudaFuncSetAttribute(qd::q_delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, qd::SMEM_ALLOC);
+  });
+  if (attr_err != cudaSuccess) {
+    set_error("refadapt_q_delta: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
+    return RA_ECUDA;
+  }
+  qd::q_delta_kernel<<<p.grid, qd::THREADS, qd::SMEM_ALLOC, static_cast<cudaStream_t>(stream)>>>(p);
   return launch_status("refadapt_q_delta");
 }
 

@@ -1,0 +1,167 @@
+"""Parity at the workloads' full sizes, through the Executor (the launch
+configuration bench.py times), on outputs the oracle can compute one by one:
+sampled O rows, sampled mass-partial tiles, every D, and the gate's decisions
+recomputed by the oracle's controller from the oracle's D."""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from _helpers import D_REL, M_ABS, TIE_BAND, bits, o_close
+
+pytestmark = pytest.mark.gpu
+
+ROLES = ("text", "ref", "tgt")
+HEADS = (0, 7, 23)
+
+
+def _wide(x):
+    return oracle.bf16_to_f64(bits(x))
+
+
+def _role(X, wl, r, z):
+    o = wl.offsets()[r]
+    return X[z, :, :, o:o + wl.n[r], :]
+
+
+def _run_stack(wl, blocks):
+    """Run the executor over `blocks` (indices into the workload's block
+    stack, as a depth-reduced stack) for all steps; returns per (t, b) the
+    inputs, outputs, D, modes, gbar and mass partials as seen after the block."""
+    from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
+    sub = synth.Workload(**{**wl.__dict__})
+    sub.n_blocks = len(blocks)
+    sub.ref_drift = [wl.ref_drift[b] for b in blocks]
+    sub.tgt_drift = [wl.tgt_drift[b] for b in blocks]
+    traj = synth.Trajectory(sub, device="cuda")
+    ex = Executor(sub.n_blocks, sub.B, sub.H, sub.d, sub.n_text, sub.n_ref, sub.n_tgt, sub.theta,
+                  sub.delta_max, sub.eps, mass_rows=sub.mass_rows, forced_boundary=sub.forced_boundary,
+                  bias=sub.bias, log_steps=sub.n_steps)
+    rec = {}
+    prev = {}
+    for t in range(sub.n_steps):
+        for b in range(sub.n_blocks):
+            X = traj.get(t, b)
+            out = {r: torch.full((sub.B, sub.H, sub.n[r], sub.d), float("nan"), dtype=torch.bfloat16,
+                                 device="cuda") for r in ROLES}
+            ex.block(t, b, roles_from_joint(X, sub.offsets(), sub.n), out)
+            torch.cuda.synchronize()
+            rec[(t, b)] = {"X": X, "O": out, "D": ex.D[b].clone(), "mode": ex.modes[t, b].clone(),
+                           "gbar": ex.gbar[t, b].clone(), "mass": ex.mass[b].clone(),
+                           "Xprev": prev.get(b)}
+            prev[b] = X
+        # keep only what later checks need
+    ex.check()
+    return sub, rec
+
+
+@pytest.mark.parametrize("name", ["c2", "c3", "c4"])
+def test_fullsize_block_parity(cuda_ok, name):
+    """First block of the stack, steps 0 and 1: sampled O rows of every
+    executed role, two mass tiles per sampled head, D of every head, and the
+    step-1 decision from the oracle controller with the oracle's D."""
+    from paper_2609_32415_gb300 import synth
+    wl = synth.make_workload(name)
+    wl.n_steps = 2
+    sub, rec = _run_stack(wl, [0])
+    sc = 1.0 / math.sqrt(sub.d)
+    bias = None if sub.bias is None else np.asarray(sub.bias)
+    rng = np.random.default_rng(0)
+    a_b = 0                                    # the cache holds step 0 after step 0's FULL
+    for t in range(2):
+        r = rec[(t, 0)]
+        mode = int(r["mode"][0])
+        if t == 0:
+            assert mode == 3
+        X = r["X"]
+        fresh_ref = mode in (2, 3)
+        Xk = X if fresh_ref else rec[(a_b, 0)]["X"]
+        hs = list(HEADS)
+        q = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 0)[0, hs]) for ro in ROLES}
+        k = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 1)[0, hs]) for ro in ROLES}
+        v = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 2)[0, hs]) for ro in ROLES}
+        keys = np.concatenate([k["text"], k["ref"], k["tgt"]], axis=1)
+        vals = np.concatenate([v["text"], v["ref"], v["tgt"]], axis=1)
+        r0, r1 = sub.n_text, sub.n_text + sub.n_ref
+        roles = ("text", "tgt") if mode == 0 else ROLES
+        for ro in roles:
+            n = sub.n[ro]
+            idx = np.unique(np.concatenate([np.arange(min(8, n)), np.arange(max(0, n - 8), n),
+                                            rng.choice(n, size=min(48, n), replace=False)]))
+            rb = np.full(len(idx), 1 if ro == "tgt" else 0, dtype=np.uint8)
+            o, _ = oracle.joint_attention(q[ro][:, idx], keys, vals, sc,
+                                          None if bias is None else bias[hs], rb if bias is not None else None,
+                                          (r0, r1))
+            got = r["O"][ro][0, hs][:, idx].double().cpu().numpy()
+            ok, worst, nw = o_close(got, o)
+            assert ok, (name, t, ro, worst, nw)
+        if mode == 0:
+            assert torch.isnan(r["O"]["ref"].float()).all()
+        # mass partials: first and last target tile of the sampled heads
+        nt = (sub.n_tgt + 127) // 128
+        base = (sub.n_text + 127) // 128
+        for tile in (0, nt - 1):
+            rows = np.arange(tile * 128, min(sub.n_tgt, tile * 128 + 128))
+            rb = np.ones(len(rows), dtype=np.uint8)
+            _, m = oracle.joint_attention(q["tgt"][:, rows], keys, vals, sc,
+                                          None if bias is None else bias[hs], rb if bias is not None else None,
+                                          (r0, r1), want_o=False)
+            got = r["mass"][0, hs, base + tile].double().cpu().numpy() / len(rows)
+            err = np.abs(got - m.mean(axis=1)).max()
+            assert err <= M_ABS, (name, t, tile, err)
+            assert err <= 2e-5, (name, t, tile, err)   # far below the gate's 1e-4 band
+        if t == 1:
+            qc = _wide(_role(X, sub, "tgt", 0)[0])
+            qp = _wide(_role(r["Xprev"], sub, "tgt", 0)[0])
+            D = oracle.q_change(qc, qp, sub.eps)
+            got = r["D"][0].double().cpu().numpy()
+            assert (np.abs(got - D) / D).max() <= D_REL
+            # the controller's decision from the oracle D and the mass of step 0
+            # (the GPU's M, whose sampled tiles were checked above at step 0)
+            M_prev = rec[(0, 0)]["mass"][0].double().sum(-1).cpu().numpy() / sub.n_tgt
+            gate = oracle.Gate(1, sub.theta, sub.delta_max, sub.forced_boundary)
+            gate.begin_step(0)
+            gate.decide(0, 0)
+            gate.begin_step(1)
+            modes, gbar = gate.decide(1, 0, D[None], M_prev[None],
+                                      tie=lambda tt, bb, s: mode == 1, tie_band=TIE_BAND)
+            assert modes[0] == mode, (name, modes, mode, gbar, sub.theta)
+            assert abs(gbar[0] - float(r["gbar"][0])) < 1e-5 * max(1.0, abs(gbar[0]))
+
+
+def test_fullsize_depth_reduced_trajectory(cuda_ok):
+    """Image-edit workload on the depth-reduced stack {0, 1, 44, 45, 59}, all 8
+    steps: every D against the oracle, every decision against the oracle's
+    controller fed with the oracle's D (and the GPU's M), and the schedule's
+    shape (full steps, monotone suffix)."""
+    from paper_2609_32415_gb300 import synth
+    wl = synth.make_workload("c2")
+    blocks = [0, 1, 44, 45, 59]
+    sub, rec = _run_stack(wl, blocks)
+    gate = oracle.Gate(1, sub.theta, sub.delta_max, sub.forced_boundary)
+    for t in range(sub.n_steps):
+        gate.begin_step(t)
+        gm = [int(rec[(t, b)]["mode"][0]) for b in range(len(blocks))]
+        for b in range(len(blocks)):
+            r = rec[(t, b)]
+            if t >= 1:
+                qc = _wide(_role(r["X"], sub, "tgt", 0)[0])
+                qp = _wide(_role(r["Xprev"], sub, "tgt", 0)[0])
+                D = oracle.q_change(qc, qp, sub.eps)
+                got = r["D"][0].double().cpu().numpy()
+                assert (np.abs(got - D) / D).max() <= D_REL, (t, b)
+                M_prev = rec[(t - 1, b)]["mass"][0].double().sum(-1).cpu().numpy() / sub.n_tgt
+                m, _ = gate.decide(t, b, D[None], M_prev[None],
+                                   tie=lambda tt, bb, s: gm[bb] == 1, tie_band=TIE_BAND)
+            else:
+                m, _ = gate.decide(t, b)
+            assert m[0] == gm[b], (t, b, m, gm)
+        if t in (0, 4):
+            assert gm == [3] * len(blocks)
+        elif 1 in gm:
+            k = gm.index(1)
+            assert gm[:k] == [0] * k and gm[k + 1:] == [2] * (len(gm) - k - 1)
+        else:
+            assert gm == [0] * len(blocks)
