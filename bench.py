@@ -49,6 +49,7 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-refresh-baseline", action="store_true")
+    ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     ap.add_argument("--sweep", action="store_true",
                     help="time the sweep workload grid (tokens x reference fraction x reuse fraction); "
@@ -287,6 +288,34 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
     return res
 
 
+def time_graphs(wl, inputs, warmup, steps):
+    """The same trajectory with every denoising step captured once as a CUDA
+    graph (one graph per trajectory step) and replayed."""
+    import torch
+    from paper_2609_32415_gb300 import Executor, roles_from_joint
+    T = wl.n_steps
+    ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max, wl.eps,
+                  mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T)
+    views = [[roles_from_joint(inputs[t][b], wl.offsets(), wl.n) for b in range(wl.n_blocks)] for t in range(T)]
+    for t in range(T):                            # eager pass: first-call set-up of every entry point
+        ex.step(t, views[t])
+    torch.cuda.synchronize()
+    graphs = [ex.capture_step(t, views[t]) for t in range(T)]
+    for i in range(warmup):
+        graphs[i % T].replay()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record()
+    for k in range(steps):
+        graphs[(warmup + k) % T].replay()
+    e1.record()
+    torch.cuda.synchronize()
+    ex.check()
+    modes = ex.modes.cpu().numpy()
+    del graphs, ex
+    return {"ms_per_step": e0.elapsed_time(e1) / steps, "modes": modes}
+
+
 def time_e2e(wl, inputs, warmup, steps):
     """Same steps through the public API with host-resident inputs: every block's
     Q/K/V are copied from pinned host memory on a copy stream (double-buffered,
@@ -506,6 +535,12 @@ def main_ours(args):
     if not args.no_refresh_baseline:
         refresh = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1, barrier=barrier)
     qd = time_q_delta(wl, inputs)
+    graph = None
+    if not args.no_graph:
+        try:
+            graph = time_graphs(wl, inputs, args.warmup, args.steps)
+        except Exception as exc:
+            graph = {"ms_per_step": None, "error": str(exc)[:200]}
     e2e = None
     if not args.no_e2e:
         try:
@@ -573,6 +608,12 @@ def main_ours(args):
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
+    if graph is not None:
+        line["cuda_graph_ms_per_step"] = None if graph.get("ms_per_step") is None else round(graph["ms_per_step"], 3)
+        if graph.get("error"):
+            line["cuda_graph_error"] = graph["error"]
+        elif "modes" in graph:
+            line["cuda_graph_modes_match"] = bool((graph["modes"] == main["modes"]).all())
     if refresh is not None:
         rms = refresh["total_ms"] / args.steps
         line["always_refresh_ms_per_step"] = round(rms, 3)

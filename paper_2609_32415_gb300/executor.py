@@ -106,5 +106,18 @@ class Executor:
             if after_block is not None:
                 after_block(t, b)
 
+    def capture_step(self, t, inputs, outs=None, log_index=None):
+        """Capture step t (every block's launches, on one stream) as a CUDA graph.
+
+        Steps must be captured in trajectory order (the Q change of step t
+        reads the target Q handed to step t-1). Capturing runs nothing;
+        replaying the graph enqueues the step with the pointers and step index
+        baked in. Make one eager call of each entry point first (first calls
+        set kernel attributes and look up driver entry points)."""
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.step(t, inputs, outs, log_index)
+        return g
+
     def check(self, stream=None):
         api.refadapt_check_error(self.err, stream)
