@@ -154,6 +154,25 @@ class Clocks:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def reduce_max_ms(local_ms, device="cpu"):
+    """Max over ranks of a per-rank timed region (the job's time), on whatever
+    process group is initialised; the local value when running alone."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(local_ms)
+    t = torch.tensor([float(local_ms)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_ms_per_step(max_total_ms, steps, world_size):
+    """Whole-job ms per denoising step: every rank runs `steps` steps of its own
+    trajectory (weak scaling), so the job completes steps x world_size steps in
+    the slowest rank's time."""
+    return max_total_ms / (steps * world_size)
+
+
 def dist_env():
     ws = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -526,11 +545,8 @@ def main_ours(args):
     clocks = Clocks(local)
     main = time_trajectory(wl, inputs, args.warmup, args.steps, attn_timing=True, clocks=clocks,
                            barrier=barrier)
-    total = torch.tensor([main["total_ms"]], dtype=torch.float64, device="cuda")
-    if ws > 1:
-        dist.all_reduce(total, op=dist.ReduceOp.MAX)
-    total_ms = float(total.item())
-    ms_per_step = total_ms / (args.steps * ws)
+    total_ms = reduce_max_ms(main["total_ms"], device="cuda")
+    ms_per_step = job_ms_per_step(total_ms, args.steps, ws)
     refresh = None
     if not args.no_refresh_baseline:
         refresh = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1, barrier=barrier)
