@@ -54,6 +54,9 @@ def parse_args():
     ap.add_argument("--sweep", action="store_true",
                     help="time the sweep workload grid (tokens x reference fraction x reuse fraction); "
                          "one JSON line per point")
+    ap.add_argument("--ablation", action="store_true",
+                    help="time the controller-cue variants (product, change, exposure, anchor x exposure, "
+                         "fixed interval 3) on the workload; one JSON line per variant")
     ap.add_argument("--blocks", type=int, default=0,
                     help="run only the first N blocks of the stack (small profiling cases)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file")
@@ -240,14 +243,15 @@ def make_inputs(wl, device):
 
 
 def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False, clocks=None,
-                    barrier=None):
+                    barrier=None, cue="product", theta=None):
     """Run warmup + timed steps (cycling the trajectory); returns timing dict."""
     import torch
     from paper_2609_32415_gb300 import Executor, roles_from_joint
     dm = wl.delta_max if delta_max is None else delta_max
-    ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, dm, wl.eps,
+    th = wl.theta if theta is None else theta
+    ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, th, dm, wl.eps,
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
-                  log_steps=wl.n_steps)
+                  log_steps=wl.n_steps, cue=cue)
     views = [[roles_from_joint(inputs[t][b], wl.offsets(), wl.n) for b in range(wl.n_blocks)]
              for t in range(wl.n_steps)]
     T = wl.n_steps
@@ -725,8 +729,49 @@ def main_sweep(args):
                 f.write(json.dumps(line) + "\n")
 
 
+def main_ablation(args):
+    """Controller ablation (paper Sec. 5.3, Tab. 4) on a synthetic trajectory:
+    the trigger cue changes, everything else (executor, stopping rule,
+    bounded-age fallback, threshold) is shared; Fixed R3 refreshes every 3 steps
+    and reuses otherwise. Reports ms per step, speedup over full computation
+    and the fraction of reusing block-steps."""
+    import torch
+    import __graft_entry__ as ge
+    from paper_2609_32415_gb300 import synth
+    ge.build()
+    wl = synth.make_workload(args.config)
+    if args.blocks > 0:
+        wl.n_blocks = min(wl.n_blocks, args.blocks)
+        wl.ref_drift, wl.tgt_drift = wl.ref_drift[:wl.n_blocks], wl.tgt_drift[:wl.n_blocks]
+    inputs = make_inputs(wl, "cuda")
+    full = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1)
+    variants = [("product", "product", None, None), ("change", "change", None, None),
+                ("exposure", "exposure", None, None), ("anchor_q_x_exposure", "anchor_product", None, None),
+                ("fixed_r3", "product", float("inf"), 3)]
+    lines = []
+    for name, cue, theta, dm in variants:
+        r = time_trajectory(wl, inputs, args.warmup, args.steps, cue=cue, theta=theta, delta_max=dm)
+        reuse = float((r["modes"][1:] == 0).mean())
+        line = {"workload": args.config, "variant": name, "theta": wl.theta if theta is None else theta,
+                "ms_per_step": round(r["total_ms"] / args.steps, 3),
+                "full_computation_ms_per_step": round(full["total_ms"] / args.steps, 3),
+                "speedup_vs_full": round(full["total_ms"] / r["total_ms"], 3),
+                "reuse_fraction_steps_1_on": round(reuse, 3)}
+        print(json.dumps(line), flush=True)
+        lines.append(line)
+    if args.out:
+        with open(args.out, "w") as f:
+            for line in lines:
+                f.write(json.dumps(line) + "\n")
+    del inputs
+    torch.cuda.empty_cache()
+
+
 def main():
     args = parse_args()
+    if args.ablation:
+        main_ablation(args)
+        return
     if args.sweep:
         main_sweep(args)
         return

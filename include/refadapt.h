@@ -191,6 +191,14 @@ ra_status refadapt_state_init(ra_state* state, int32_t B, void* stream);
  * else BOUNDARY (and latch) if gbar >= theta — or b >= forced_boundary when
  * forced_boundary >= 0 — else REUSE.
  *
+ * cue selects the per-head trigger of the controller ablation (paper Sec. 5.3,
+ * Tab. 4; App. A.2), everything else unchanged: RA_CUE_PRODUCT g_h = D_h M_h
+ * (the method), RA_CUE_CHANGE g_h = D_h (target-Q change only),
+ * RA_CUE_EXPOSURE g_h = M_h (exposure only). The anchor-relative variant is
+ * RA_CUE_PRODUCT fed with the change to the block's last materialisation
+ * (c^anchor of App. A.2) in q_delta; the fixed-interval baseline is
+ * theta = +inf with delta_max = the interval.
+ *
  *  q_delta            device [B][H] (refadapt_q_delta for this step/block);
  *                     may be NULL at t == 0.
  *  mass_partial_prev  device [B][H][mass_partial_len] from step t-1, block b;
@@ -209,6 +217,8 @@ typedef struct {
   int32_t forced_boundary;
   int32_t mass_partial_len;
   int32_t mass_row_count;
+  int32_t cue;         /* ra_cue */
+  int32_t reserved;    /* set to 0 */
   const float* q_delta;
   const float* mass_partial_prev;
   ra_state* state;
@@ -216,6 +226,8 @@ typedef struct {
   float* gbar_out;
   float* m_out;
 } ra_gate_args;
+
+typedef enum { RA_CUE_PRODUCT = 0, RA_CUE_CHANGE = 1, RA_CUE_EXPOSURE = 2 } ra_cue;
 
 ra_status refadapt_gate(const ra_gate_args* args, void* stream);
 

@@ -158,9 +158,18 @@ class Gate:
     with theta (Eq. 13): below theta the block reuses, the first block at or
     above theta is the boundary and sets the latch; every later block computes.
     ``forced_boundary`` >= 0 replaces the comparison by "block index >= it".
+    ``cue`` selects the per-head trigger of the controller ablation (Sec. 5.3,
+    Tab. 4): "product" g_h = D_h M_h (the method), "change" g_h = D_h,
+    "exposure" g_h = M_h. Only the trigger changes; the executor, stopping
+    rule, bounded-age fallback and threshold stay.
     """
 
-    def __init__(self, n_samples, theta, delta_max, forced_boundary=-1):
+    CUES = ("product", "change", "exposure")
+
+    def __init__(self, n_samples, theta, delta_max, forced_boundary=-1, cue="product"):
+        if cue not in self.CUES:
+            raise ValueError("unknown cue %r" % (cue,))
+        self.cue = cue
         self.B = int(n_samples)
         self.theta = float(theta)
         self.delta_max = int(delta_max)
@@ -191,7 +200,12 @@ class Gate:
         modes, gbars = [], []
         for s in range(self.B):
             if t >= 1 and D is not None and M_prev is not None:
-                g = [float(D[s][h]) * float(M_prev[s][h]) for h in range(len(D[s]))]
+                if self.cue == "change":
+                    g = [float(D[s][h]) for h in range(len(D[s]))]
+                elif self.cue == "exposure":
+                    g = [float(M_prev[s][h]) for h in range(len(D[s]))]
+                else:
+                    g = [float(D[s][h]) * float(M_prev[s][h]) for h in range(len(D[s]))]
                 gbar = sum(g) / len(g)
             else:
                 gbar = float("nan")
@@ -269,7 +283,7 @@ def block_attention(q, k, v, mode, scale, bias=None, mass_rows=0, o_rows=None,
 
 def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
                 scale=None, bias=None, mass_rows=0, forced_boundary=-1, tie=None,
-                o_rows=None, want_o=True, nthreads=None):
+                o_rows=None, want_o=True, nthreads=None, cue="product"):
     """Algorithm 1 over ``n_steps`` denoising steps and ``n_blocks`` blocks.
 
     ``get_inputs(t, b)`` returns dict role -> (q, k, v), each a uint16 array of
@@ -286,10 +300,16 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
     K/V/Q and a_b = t, then every row runs. D and M are recorded at every block
     for the next step.
 
+    ``cue``: "product" (the method), "change", "exposure" (Tab. 4 variants),
+    or "anchor_product": g_h = c^anchor_h M_h with c^anchor the change of the
+    target query to its value at the block's last materialisation a_b
+    (App. A.2), i.e. Eq. 1 against the anchor instead of the previous step.
+
     Returns records[t][b] = dict(mode [B], gbar [B], D [B,H], M [B,H],
     O [B] of dict role -> array or None, a_b [B]).
     """
-    gate = Gate(B, theta, delta_max, forced_boundary)
+    gate = Gate(B, theta, delta_max, forced_boundary, "product" if cue == "anchor_product" else cue)
+    anchor_q = [None] * n_blocks                       # target Q at the last materialisation
     cache = [[None] * B for _ in range(n_blocks)]      # dict(k, v, q) per block/sample
     a_b = [[-1] * B for _ in range(n_blocks)]
     prev_q = [None] * n_blocks                         # target Q, float64 [B,H,n,d]
@@ -304,8 +324,16 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
             q_tgt = f["tgt"][0]
             H, d = q_tgt.shape[1], q_tgt.shape[3]
             sc = (1.0 / math.sqrt(d)) if scale is None else float(scale)
-            D = q_change(q_tgt, prev_q[b], eps) if (t >= 1 and prev_q[b] is not None) else None
+            if cue == "anchor_product":
+                D = q_change(q_tgt, anchor_q[b], eps) if (t >= 1 and anchor_q[b] is not None) else None
+            else:
+                D = q_change(q_tgt, prev_q[b], eps) if (t >= 1 and prev_q[b] is not None) else None
             modes, gbars = gate.decide(t, b, D, prev_M[b], tie=tie)
+            if anchor_q[b] is None:
+                anchor_q[b] = np.array(q_tgt)
+            for s in range(B):
+                if modes[s] in (COMPUTE, FULL):
+                    anchor_q[b][s] = q_tgt[s]
             M = np.zeros((B, H))
             O = []
             for s in range(B):

@@ -13,6 +13,7 @@ LIB_PATH = os.path.join(PKG, "librefadapt.so")
 RA_OK, RA_EINVAL, RA_EUNSUPPORTED, RA_ECUDA, RA_ETIMEOUT = 0, 1, 2, 3, 4
 RA_MODE_REUSE, RA_MODE_BOUNDARY, RA_MODE_COMPUTE, RA_MODE_FULL = 0, 1, 2, 3
 RA_TEXT, RA_REF, RA_TGT = 0, 1, 2
+RA_CUE_PRODUCT, RA_CUE_CHANGE, RA_CUE_EXPOSURE = 0, 1, 2
 RA_MASS_TILE_ROWS = 128
 RA_Q_DELTA_NOALLOC_MAX_BH = 96
 
@@ -41,7 +42,8 @@ class RaAttnArgs(ctypes.Structure):
 class RaGateArgs(ctypes.Structure):
     _fields_ = [("theta", c_double), ("t", c_int32), ("b", c_int32), ("B", c_int32), ("H", c_int32),
                 ("delta_max", c_int32), ("forced_boundary", c_int32), ("mass_partial_len", c_int32),
-                ("mass_row_count", c_int32), ("q_delta", c_void_p), ("mass_partial_prev", c_void_p),
+                ("mass_row_count", c_int32), ("cue", c_int32), ("reserved", c_int32),
+                ("q_delta", c_void_p), ("mass_partial_prev", c_void_p),
                 ("state", c_void_p), ("mode_out", c_void_p), ("gbar_out", c_void_p),
                 ("m_out", c_void_p)]
 

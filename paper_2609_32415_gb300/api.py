@@ -114,7 +114,7 @@ def new_state(B, device="cuda", stream=None):
 
 
 def refadapt_gate(t, b, state, mode_out, theta, delta_max, B, H, q_delta=None, mass_partial_prev=None,
-                  mass_row_count=0, forced_boundary=-1, gbar_out=None, m_out=None, stream=None):
+                  mass_row_count=0, forced_boundary=-1, gbar_out=None, m_out=None, cue=0, stream=None):
     a = RaGateArgs()
     a.theta = float(theta)
     a.t, a.b, a.B, a.H = int(t), int(b), int(B), int(H)
@@ -122,6 +122,7 @@ def refadapt_gate(t, b, state, mode_out, theta, delta_max, B, H, q_delta=None, m
     a.forced_boundary = int(forced_boundary)
     a.mass_partial_len = int(mass_partial_prev.shape[-1]) if mass_partial_prev is not None else 0
     a.mass_row_count = int(mass_row_count)
+    a.cue = int(cue)
     a.q_delta = _ptr(q_delta)
     a.mass_partial_prev = _ptr(mass_partial_prev)
     a.state = _ptr(state)

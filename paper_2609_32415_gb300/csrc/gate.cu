@@ -1,7 +1,8 @@
 // refadapt_gate: Algorithm 1's per-block decision on the device, so a whole
 // denoising step can be enqueued (or graph-captured) without a host sync.
 //
-// Score (paper Eq. 12): g_{t,b,h} = D_{t,b,h} * M_{t-1,b,h}, formed per head;
+// Score (paper Eq. 12): g_{t,b,h} = D_{t,b,h} * M_{t-1,b,h}, formed per head
+// (or D alone / M alone for the controller ablation of Sec. 5.3);
 // aggregate (App. A.2): gbar = mean_h g; cutoff (Eq. 13): the first block with
 // gbar >= theta reactivates, deeper blocks compute; bounded-age refresh
 // (Sec. 4): t - a_full >= delta_max recomputes every block of the step.
@@ -29,7 +30,7 @@ constexpr int THREADS = 256;
 
 struct Params {
   double theta;
-  int32_t t, b, B, H, delta_max, forced_boundary, mpl, mass_rows_count;
+  int32_t t, b, B, H, delta_max, forced_boundary, mpl, mass_rows_count, cue;
   const float* qd;
   const float* mp;
   ra_state* st;
@@ -98,8 +99,12 @@ __global__ void __launch_bounds__(THREADS) gate_kernel(const Params p) {
     }
     const bool have = (p.t >= 1) && p.qd && p.mp;
     double gsum = 0.0;
-    if (have)
-      for (int h = 0; h < p.H; ++h) gsum += double(p.qd[s * p.H + h]) * m_sh[s * p.H + h];
+    if (have) {
+      for (int h = 0; h < p.H; ++h) {
+        const double dh = double(p.qd[s * p.H + h]), mh = m_sh[s * p.H + h];
+        gsum += (p.cue == RA_CUE_CHANGE) ? dh : (p.cue == RA_CUE_EXPOSURE) ? mh : dh * mh;
+      }
+    }
     const double gbar = have ? gsum / double(p.H) : NAN;
     if (p.gbar_out) p.gbar_out[s] = float(gbar);
     int32_t mode;
@@ -167,6 +172,10 @@ extern "C" ra_status refadapt_gate(const ra_gate_args* a, void* stream) {
     set_error("refadapt_gate: B * H must be <= 6144");
     return RA_EINVAL;
   }
+  if (a->cue != RA_CUE_PRODUCT && a->cue != RA_CUE_CHANGE && a->cue != RA_CUE_EXPOSURE) {
+    set_error("refadapt_gate: unknown cue %d", a->cue);
+    return RA_EINVAL;
+  }
   if (std::isnan(a->theta)) {
     set_error("refadapt_gate: theta is NaN");
     return RA_EINVAL;
@@ -181,6 +190,7 @@ extern "C" ra_status refadapt_gate(const ra_gate_args* a, void* stream) {
   p.forced_boundary = a->forced_boundary;
   p.mpl = a->mass_partial_len;
   p.mass_rows_count = a->mass_row_count;
+  p.cue = a->cue;
   p.qd = a->q_delta;
   p.mp = a->mass_partial_prev;
   p.st = a->state;

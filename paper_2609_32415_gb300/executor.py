@@ -28,10 +28,26 @@ def roles_from_joint(X, offsets, n):
     return out
 
 
+CUES = {"product": 0, "change": 1, "exposure": 2, "anchor_product": 0}
+
+
 class Executor:
+    """Algorithm 1 over a block stack.
+
+    ``cue`` picks the reactivation trigger of the controller ablation (paper
+    Sec. 5.3, Tab. 4): "product" (D x M, the method), "change" (target-Q change
+    only), "exposure" (M only), or "anchor_product" (the change of the target
+    query to its value at the block's last materialisation, App. A.2, times M;
+    the executor keeps that anchor per block). The fixed-interval baseline is
+    theta = inf with delta_max = the interval.
+    """
+
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
                  mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
-                 device="cuda"):
+                 device="cuda", cue="product"):
+        if cue not in CUES:
+            raise ValueError("unknown cue %r" % (cue,))
+        self.cue = cue
         self.n_blocks, self.B, self.H, self.d = n_blocks, B, H, d
         self.n = {"text": n_text, "ref": n_ref, "tgt": n_tgt}
         self.theta, self.delta_max, self.eps = float(theta), int(delta_max), float(eps)
@@ -56,6 +72,8 @@ class Executor:
         self.state = api.new_state(B, dev)
         self.err = torch.zeros(1, dtype=torch.int32, device=dev)
         self._prev_qtgt = [None] * n_blocks
+        self.anchor = (torch.zeros((n_blocks, B, H, n_tgt, d), dtype=torch.bfloat16, device=dev)
+                       if cue == "anchor_product" else None)
         self._out = None
         self.attn_hook = None   # optional callable(phase in {"pre", "post"}, t, b), e.g. CUDA events
 
@@ -74,12 +92,18 @@ class Executor:
         qt = x["tgt"][0]
         have_prev = t >= 1 and self._prev_qtgt[b] is not None
         if have_prev:
-            api.refadapt_q_delta(qt, self._prev_qtgt[b], self.D[b], self.workspace, self.eps, stream)
+            ref_q = self.anchor[b] if self.anchor is not None else self._prev_qtgt[b]
+            api.refadapt_q_delta(qt, ref_q, self.D[b], self.workspace, self.eps, stream)
         api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
                           q_delta=self.D[b] if have_prev else None,
                           mass_partial_prev=self.mass[b] if have_prev else None,
                           mass_row_count=self.mass_row_count, forced_boundary=self.forced_boundary,
-                          gbar_out=self.gbar[li, b], m_out=self.M[li, b], stream=stream)
+                          gbar_out=self.gbar[li, b], m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
+        if self.anchor is not None:
+            # Materialising blocks move their anchor to this step's target Q (the
+            # V copy is skipped: source and destination coincide).
+            an = self.anchor[b]
+            api.refadapt_ref_cache_update(qt, an, an, an, mode, t, None, stream=stream)
         qr, kr, vr = x["ref"]
         api.refadapt_ref_cache_update(kr, vr, self.cache_k[b], self.cache_v[b], mode, t, self.a_b[b],
                                       x_src=qr, x_cache=self.cache_x[b], stream=stream)

@@ -12,12 +12,12 @@ pytestmark = pytest.mark.gpu
 ROLES = ("text", "ref", "tgt")
 
 
-def _run_both(wl, o_sample=None):
+def _run_both(wl, o_sample=None, cue="product"):
     from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
     traj = synth.Trajectory(wl, device="cuda")
     ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max,
                   wl.eps, mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
-                  log_steps=wl.n_steps)
+                  log_steps=wl.n_steps, cue=cue)
     keep, outs, D = {}, {}, np.zeros((wl.n_steps, wl.n_blocks, wl.B, wl.H))
     for t in range(wl.n_steps):
         xs, os_ = [], []
@@ -49,7 +49,7 @@ def _run_both(wl, o_sample=None):
 
     rec = oracle.closed_loop(raw, wl.n_steps, wl.n_blocks, wl.B, theta=wl.theta, delta_max=wl.delta_max,
                              eps=wl.eps, bias=wl.bias, mass_rows=wl.mass_rows,
-                             forced_boundary=wl.forced_boundary, tie=tie, o_rows=o_sample)
+                             forced_boundary=wl.forced_boundary, tie=tie, o_rows=o_sample, cue=cue)
     return modes, gbar, Mlog, D, outs, rec
 
 
@@ -111,3 +111,14 @@ def test_closed_loop_forced_boundary_and_bias(cuda_ok):
     res = _run_both(wl)
     _compare(wl, *res)
     assert list(res[0][1, :, 0]) == [0, 0, 1, 2]
+
+
+@pytest.mark.parametrize("cue,theta", [("change", 0.15), ("exposure", 0.43), ("anchor_product", 0.1)])
+def test_closed_loop_ablation_cues(cuda_ok, cue, theta):
+    """The controller ablation's trigger variants (Sec. 5.3, Tab. 4; the anchor
+    variant of App. A.2) through the same executor."""
+    from paper_2609_32415_gb300 import synth
+    wl = synth.custom_workload(2, 4, 128, 33, 300, 200, n_blocks=5, n_steps=6, ref_drift=0.05,
+                               tgt_drift=[0.05, 0.1, 0.2, 0.3, 0.4], theta=theta, delta_max=4)
+    res = _run_both(wl, cue=cue)
+    _compare(wl, *res)

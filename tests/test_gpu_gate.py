@@ -11,7 +11,10 @@ from _helpers import TIE_BAND
 pytestmark = pytest.mark.gpu
 
 
-def _run_gate(D, M, theta, delta_max, forced=-1, L=3):
+CUE_ID = {"product": 0, "change": 1, "exposure": 2}
+
+
+def _run_gate(D, M, theta, delta_max, forced=-1, L=3, cue="product"):
     """D, M: [T, nb, B, H] arrays. M is spread over L partial tiles. Returns GPU
     modes / gbar [T, nb, B] and the oracle's."""
     from paper_2609_32415_gb300 import api
@@ -35,13 +38,14 @@ def _run_gate(D, M, theta, delta_max, forced=-1, L=3):
             prev = mparts[(t - 1) * nb + b] if t >= 1 else None
             api.refadapt_gate(t, b, state, modes[t, b], theta, delta_max, B, H,
                               q_delta=dd[t, b] if t >= 1 else None, mass_partial_prev=prev,
-                              mass_row_count=rows, forced_boundary=forced, gbar_out=gbar[t, b])
+                              mass_row_count=rows, forced_boundary=forced, gbar_out=gbar[t, b],
+                              cue=CUE_ID[cue])
     torch.cuda.synchronize()
     gm = modes.cpu().numpy()
     gg = gbar.double().cpu().numpy()
     # Oracle, using the M the GPU sees (the float32 partial sums) and the float32 D.
     Mq = np.stack([m.double().sum(-1).cpu().numpy() / rows for m in mparts]).reshape(T, nb, B, H)
-    gate = oracle.Gate(B, theta, delta_max, forced)
+    gate = oracle.Gate(B, theta, delta_max, forced, cue)
     om = np.zeros((T, nb, B), dtype=np.int32)
     og = np.zeros((T, nb, B))
     for t in range(T):
@@ -92,3 +96,16 @@ def test_gate_bounded_age(cuda_ok):
     assert np.array_equal(gm, om)
     for t in range(T):
         assert np.all(gm[t] == (3 if t % 3 == 0 else 0))
+
+
+@pytest.mark.parametrize("cue,theta", [("change", 0.3), ("exposure", 0.45)])
+def test_gate_ablation_cues(cuda_ok, cue, theta):
+    """Sec. 5.3 / Tab. 4 trigger variants: D alone or M alone, same controller."""
+    rng = np.random.default_rng(7)
+    T, nb, B, H = 6, 10, 2, 24
+    D = rng.uniform(0.0, 0.6, size=(T, nb, B, H))
+    M = rng.uniform(0.0, 0.9, size=(T, nb, B, H))
+    gm, gg, om, og = _run_gate(D, M, theta=theta, delta_max=4, cue=cue)
+    assert np.array_equal(gm, om)
+    fin = np.isfinite(og)
+    np.testing.assert_allclose(gg[fin], og[fin], rtol=1e-6, atol=1e-7)

@@ -389,3 +389,52 @@ def test_boundary_uses_cached_reference_kv():
     o, _ = _plain_block(mixed, 0, 1 / math.sqrt(8))
     got = np.concatenate([rec[1][0]["O"][0][r] for r in oracle.ROLES], axis=1)
     np.testing.assert_allclose(got, o, rtol=0, atol=1e-14)
+
+
+# --------------------------------------------------------------------------- controller ablation cues
+def test_gate_cues_change_and_exposure():
+    """Sec. 5.3 / Tab. 4: only the trigger changes; D alone or M alone per head."""
+    D = [[0.3, 0.1]]
+    M = [[0.5, 0.9]]
+    for cue, want in (("product", (0.15 + 0.09) / 2), ("change", 0.2), ("exposure", 0.7)):
+        g = oracle.Gate(1, 0.19, 100, cue=cue)
+        g.begin_step(1)
+        modes, gbar = g.decide(1, 0, D, M)
+        assert gbar[0] == pytest.approx(want, abs=1e-15)
+        assert modes[0] == (BOUNDARY if want >= 0.19 else REUSE)
+    with pytest.raises(ValueError):
+        oracle.Gate(1, 0.1, 4, cue="bogus")
+
+
+def test_anchor_cue_measures_change_to_last_materialisation():
+    """App. A.2: c^anchor = ||Q_t - Q_{a_b}|| / (||Q_{a_b}|| + eps). With theta = inf
+    no block rematerialises after step 0, so the anchor stays at step 0."""
+    traj = _tiny_inputs(ref_drift=0.1, tgt_drift=0.2, seed=8)
+    rec = oracle.closed_loop(lambda t, b: traj[(t, b)], 4, 3, 2, theta=math.inf, delta_max=10 ** 6,
+                             cue="anchor_product")
+    for t in range(1, 4):
+        for b in range(3):
+            q0 = oracle.bf16_to_f64(traj[(0, b)]["tgt"][0])
+            qt = oracle.bf16_to_f64(traj[(t, b)]["tgt"][0])
+            np.testing.assert_allclose(rec[t][b]["D"], oracle.q_change(qt, q0), rtol=0, atol=1e-15)
+    # consecutive-change cue for comparison: D_t is against step t-1
+    rec2 = oracle.closed_loop(lambda t, b: traj[(t, b)], 4, 3, 2, theta=math.inf, delta_max=10 ** 6,
+                              cue="change")
+    q1 = oracle.bf16_to_f64(traj[(1, 0)]["tgt"][0])
+    q2 = oracle.bf16_to_f64(traj[(2, 0)]["tgt"][0])
+    np.testing.assert_allclose(rec2[2][0]["D"], oracle.q_change(q2, q1), rtol=0, atol=1e-15)
+
+
+def test_anchor_moves_with_materialisation():
+    """theta = 0: block 0 is the boundary every step (its anchor stays at step 0),
+    blocks 1, 2 compute every step (their anchor is the previous step)."""
+    traj = _tiny_inputs(ref_drift=0.1, tgt_drift=0.2, seed=9)
+    rec = oracle.closed_loop(lambda t, b: traj[(t, b)], 4, 3, 2, theta=0.0, delta_max=10 ** 6,
+                             cue="anchor_product")
+    for t in range(2, 4):
+        q = {k: oracle.bf16_to_f64(traj[(k, b)]["tgt"][0]) for k in range(4) for b in [0]}
+        np.testing.assert_allclose(rec[t][0]["D"], oracle.q_change(q[t], q[0]), atol=1e-15)
+        for b in (1, 2):
+            qt = oracle.bf16_to_f64(traj[(t, b)]["tgt"][0])
+            qp = oracle.bf16_to_f64(traj[(t - 1, b)]["tgt"][0])
+            np.testing.assert_allclose(rec[t][b]["D"], oracle.q_change(qt, qp), atol=1e-15)
