@@ -57,6 +57,8 @@ def parse_args():
     ap.add_argument("--ablation", action="store_true",
                     help="time the controller-cue variants (product, change, exposure, anchor x exposure, "
                          "fixed interval 3) on the workload; one JSON line per variant")
+    ap.add_argument("--diagnostics", action="store_true",
+                    help="also time the trajectory with the staleness diagnostics on (every 8th target row)")
     ap.add_argument("--blocks", type=int, default=0,
                     help="run only the first N blocks of the stack (small profiling cases)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file")
@@ -243,7 +245,7 @@ def make_inputs(wl, device):
 
 
 def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False, clocks=None,
-                    barrier=None, cue="product", theta=None):
+                    barrier=None, cue="product", theta=None, diagnostics=False, diag_row_stride=8):
     """Run warmup + timed steps (cycling the trajectory); returns timing dict."""
     import torch
     from paper_2609_32415_gb300 import Executor, roles_from_joint
@@ -251,7 +253,7 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
     th = wl.theta if theta is None else theta
     ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, th, dm, wl.eps,
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
-                  log_steps=wl.n_steps, cue=cue)
+                  log_steps=wl.n_steps, cue=cue, diagnostics=diagnostics, diag_row_stride=diag_row_stride)
     views = [[roles_from_joint(inputs[t][b], wl.offsets(), wl.n) for b in range(wl.n_blocks)]
              for t in range(wl.n_steps)]
     T = wl.n_steps
@@ -555,6 +557,9 @@ def main_ours(args):
     if not args.no_refresh_baseline:
         refresh = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1, barrier=barrier)
     qd = time_q_delta(wl, inputs)
+    diag = None
+    if args.diagnostics:
+        diag = time_trajectory(wl, inputs, args.warmup, args.steps, diagnostics=True, diag_row_stride=8)
     graph = None
     if not args.no_graph:
         try:
@@ -628,6 +633,10 @@ def main_ours(args):
         "e2e": e2e,
         "cpu_baseline": cpu,
     }
+    if diag is not None:
+        dms = diag["total_ms"] / args.steps
+        line["diagnostics_ms_per_step"] = round(dms, 3)
+        line["diagnostics_overhead"] = round(dms / (main["total_ms"] / args.steps) - 1.0, 4)
     if graph is not None:
         line["cuda_graph_ms_per_step"] = None if graph.get("ms_per_step") is None else round(graph["ms_per_step"], 3)
         if graph.get("error"):

@@ -89,7 +89,8 @@ typedef struct {
  * the softmax probability summed over reference keys, l_ref(q) / l(q), is
  * accumulated per 128-row Q tile into mass_partial[b][h][i] (fp32), i over
  * the text tiles (ceil(n_text/128)) then the target tiles
- * (ceil(n_tgt/128)); refadapt_mass_partial_len() gives the length. Mass row
+ * (ceil(n_tgt/128)), n counting query rows; refadapt_mass_partial_len()
+ * gives the length. Mass row
  * set: target rows (mass_rows = 0), or text + target rows (mass_rows = 1);
  * partials of tiles outside the set are written as 0. M_{t,b,h} is the sum of
  * a (b, h) row of partials divided by the number of mass rows (the gate does
@@ -97,10 +98,13 @@ typedef struct {
  * (deterministic).
  *
  * Arguments:
- *  q, k, v, o [3]   segments per role (RA_TEXT, RA_REF, RA_TGT). For each
- *                   role all four must have the same n; n_tgt >= 1.
- *                   q[RA_REF] / o[RA_REF] may have ptr NULL only if n_ref == 0
- *                   or every sample reuses.
+ *  q, k, v, o [3]   segments per role (RA_TEXT, RA_REF, RA_TGT). Per role q
+ *                   and o share n (query rows) and k and v share n (key
+ *                   rows); query and key rows of a role may differ (e.g. a
+ *                   row sample of the queries). The target segment needs at
+ *                   least one key row. q[RA_REF] / o[RA_REF] with ptr NULL:
+ *                   the reference query rows are not computed, whatever the
+ *                   mode.
  *  B, H, d          batch, heads, head dim; d in {64, 128}.
  *  softmax_scale    > 0; pass 0 for 1/sqrt(d).
  *  ref_logit_bias   device [H] fp32 or NULL: added to the logits of target

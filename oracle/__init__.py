@@ -10,9 +10,9 @@ tests/test_oracle_pins.py against brute force, closed forms, library special
 cases and invariants; none is "parity unpinned".
 """
 from .core import (REUSE, BOUNDARY, COMPUTE, FULL, ROLES, Gate, attention_flops,
-                   bf16_to_f64, block_attention, closed_loop, default_threads, exposure,
-                   joint_attention, q_change, reuse_score_fraction)
+                   bf16_to_f64, block_attention, closed_loop, default_threads, endpoint_drift, exposure,
+                   joint_attention, local_impact, q_change, reuse_score_fraction)
 
 __all__ = ["REUSE", "BOUNDARY", "COMPUTE", "FULL", "ROLES", "Gate", "attention_flops",
-           "bf16_to_f64", "block_attention", "closed_loop", "default_threads", "exposure",
-           "joint_attention", "q_change", "reuse_score_fraction"]
+           "bf16_to_f64", "block_attention", "closed_loop", "default_threads", "endpoint_drift", "exposure",
+           "joint_attention", "local_impact", "q_change", "reuse_score_fraction"]

@@ -123,6 +123,18 @@ def q_change(q_cur, q_prev, eps=1e-6) -> np.ndarray:
     return num / den
 
 
+def endpoint_drift(z_t, z_a, eps=1e-6) -> np.ndarray:
+    """Eq. 7, D_{t|a}(Z) = ||Z_t - Z_a||_F / (||Z_a||_F + eps): anchor-to-current
+    change of a reference tensor (per leading index)."""
+    return q_change(z_t, z_a, eps)
+
+
+def local_impact(o_stale, o_fresh, eps=1e-6) -> np.ndarray:
+    """Eq. 10, I = ||O^staleKV - O^fresh||_F / (||O^fresh||_F + eps) over the
+    target query rows (per leading index)."""
+    return q_change(o_stale, o_fresh, eps)
+
+
 def exposure(row_mass_tgt, row_mass_text=None) -> np.ndarray:
     """Eq. 4: mean over the chosen query rows of their reference mass, per head.
 
@@ -283,7 +295,8 @@ def block_attention(q, k, v, mode, scale, bias=None, mass_rows=0, o_rows=None,
 
 def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
                 scale=None, bias=None, mass_rows=0, forced_boundary=-1, tie=None,
-                o_rows=None, want_o=True, nthreads=None, cue="product"):
+                o_rows=None, want_o=True, nthreads=None, cue="product", diagnostics=False,
+                diag_row_stride=1):
     """Algorithm 1 over ``n_steps`` denoising steps and ``n_blocks`` blocks.
 
     ``get_inputs(t, b)`` returns dict role -> (q, k, v), each a uint16 array of
@@ -305,8 +318,16 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
     target query to its value at the block's last materialisation a_b
     (App. A.2), i.e. Eq. 1 against the anchor instead of the previous step.
 
+    ``diagnostics``: also record, per block, the staleness diagnostics of
+    Sec. 3.3 and App. A.2 on the target rows 0, k, 2k, ... (k =
+    ``diag_row_stride``): E_K, E_V (Eq. 7: cache slot vs this step's fresh
+    reference K, V), E_KV = (E_K + E_V) / 2, O_fresh (Eq. 8: target rows with
+    fresh reference K/V), I_KV (Eq. 10: executed output vs O_fresh) and
+    M_fresh (the exposure of Eq. 4 with fresh reference keys; the executed M
+    is the same-step cached exposure when the block reuses).
+
     Returns records[t][b] = dict(mode [B], gbar [B], D [B,H], M [B,H],
-    O [B] of dict role -> array or None, a_b [B]).
+    O [B] of dict role -> array or None, a_b [B]) (+ the diagnostics).
     """
     gate = Gate(B, theta, delta_max, forced_boundary, "product" if cue == "anchor_product" else cue)
     anchor_q = [None] * n_blocks                       # target Q at the last materialisation
@@ -336,6 +357,7 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
                     anchor_q[b][s] = q_tgt[s]
             M = np.zeros((B, H))
             O = []
+            diag = {}
             for s in range(B):
                 mode = modes[s]
                 if mode in (COMPUTE, FULL):
@@ -354,9 +376,29 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
                                       mass_rows, rows, want_o, nthreads)
                 M[s] = res["M"]
                 O.append(res["O"])
-            step_rec.append({"mode": modes, "gbar": gbars,
-                             "D": None if D is None else np.asarray(D),
-                             "M": M, "O": O, "a_b": list(a_b[b])})
+                if diagnostics:
+                    k = int(diag_row_stride)
+                    qf = {"text": f["text"][0][s], "ref": f["ref"][0][s], "tgt": f["tgt"][0][s][:, ::k]}
+                    kf = {"text": f["text"][1][s], "ref": f["ref"][1][s], "tgt": f["tgt"][1][s]}
+                    vf = {"text": f["text"][2][s], "ref": f["ref"][2][s], "tgt": f["tgt"][2][s]}
+                    fresh = block_attention(qf, kf, vf, REUSE, sc, None if bias is None else np.asarray(bias),
+                                            0, None, True, nthreads)
+                    # target rows of the executed pass, same sampling
+                    qs = {"text": f["text"][0][s], "ref": qref, "tgt": f["tgt"][0][s][:, ::k]}
+                    stale = block_attention(qs, kd, vd, REUSE, sc, None if bias is None else np.asarray(bias),
+                                            0, None, True, nthreads)
+                    diag.setdefault("E_K", np.zeros((B, H)))[s] = endpoint_drift(f["ref"][1][s], kref, eps)
+                    diag.setdefault("E_V", np.zeros((B, H)))[s] = endpoint_drift(f["ref"][2][s], vref, eps)
+                    diag.setdefault("I_KV", np.zeros((B, H)))[s] = local_impact(stale["O"]["tgt"],
+                                                                               fresh["O"]["tgt"], eps)
+                    diag.setdefault("M_fresh", np.zeros((B, H)))[s] = fresh["M"]
+                    diag.setdefault("M_cached", np.zeros((B, H)))[s] = stale["M"]
+            rec = {"mode": modes, "gbar": gbars, "D": None if D is None else np.asarray(D),
+                   "M": M, "O": O, "a_b": list(a_b[b])}
+            if diagnostics:
+                diag["E_KV"] = 0.5 * (diag["E_K"] + diag["E_V"])
+                rec.update(diag)
+            step_rec.append(rec)
             prev_q[b] = q_tgt
             prev_M[b] = M
         records.append(step_rec)

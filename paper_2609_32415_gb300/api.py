@@ -58,11 +58,11 @@ def refadapt_joint_attn(q, k, v, o, mass_partial, mode=None, softmax_scale=0.0, 
     a = RaAttnArgs()
     a.B, a.H, a.d, a.mass_rows = B, H, d, int(mass_rows)
     for r in range(3):
-        n_r = k[r].shape[2]
-        a.q[r] = seg(q[r], n_r)
+        n_q = q[r].shape[2] if q[r] is not None else k[r].shape[2]
+        a.q[r] = seg(q[r], n_q)
         a.k[r] = seg(k[r])
         a.v[r] = seg(v[r])
-        a.o[r] = seg(o[r], n_r)
+        a.o[r] = seg(o[r], n_q)
     a.softmax_scale = float(softmax_scale)
     a.ref_logit_bias = _ptr(ref_logit_bias)
     a.mode = _ptr(mode)

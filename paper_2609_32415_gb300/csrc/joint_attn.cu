@@ -72,7 +72,8 @@ struct Params {
   CUtensorMap tm_v[3];
   __nv_bfloat16* o_ptr[3];
   int64_t o_sb[3], o_sh[3], o_sn[3];
-  int32_t n[3];
+  int32_t nq[3];  // query rows per role
+  int32_t nk[3];  // key rows per role
   int32_t q_tiles[3];
   int32_t q_blocks[3];  // pairs of Q tiles
   int32_t kv_tiles[3];
@@ -350,7 +351,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
     for (int j = 0; ok && j < nkv; ++j) {
       int r, row0;
       kv_tile(p, j, r, row0);
-      const int nvalid = min(BN, p.n[r] - row0);
+      const int nvalid = min(BN, p.nk[r] - row0);
       const float badd = (r == 1) ? bias_l2 : 0.f;
       ok = __all_sync(0xffffffffu, mbar_wait(s_full + t, j & 1, ctl));
       if (!ok) break;
@@ -436,7 +437,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
     }
     if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done + t, (nkv - 1) & 1, ctl));
     const int grow = tile * BM + row;
-    const bool valid = active && grow < p.n[role];
+    const bool valid = active && grow < p.nq[role];
     const float inv_l = 1.f / l;
     if (ok) {
       tc_fence_after();
@@ -538,12 +539,10 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
   char what[64];
   Params p;
   std::memset(&p, 0, sizeof(p));
-  const int n_ref = a->k[RA_REF].n;
   bool ref_rows = true;
   for (int r = 0; r < 3; ++r) {
-    const int n = a->k[r].n;
-    if (a->q[r].n != n || a->v[r].n != n || a->o[r].n != n) {
-      set_error("refadapt_joint_attn: %s segments disagree on n", names[r]);
+    if (a->v[r].n != a->k[r].n || a->o[r].n != a->q[r].n) {
+      set_error("refadapt_joint_attn: %s: k and v (key rows) or q and o (query rows) disagree on n", names[r]);
       return RA_EINVAL;
     }
     const ra_seg* segs[4] = {&a->q[r], &a->k[r], &a->v[r], &a->o[r]};
@@ -559,35 +558,31 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
     }
   }
   if (a->k[RA_TGT].n < 1) {
-    set_error("refadapt_joint_attn: n_tgt must be >= 1");
+    set_error("refadapt_joint_attn: the target segment needs at least one key row");
     return RA_EINVAL;
   }
   const int d = a->d;
   for (int r = 0; r < 3; ++r) {
-    const int n = a->k[r].n;
-    p.n[r] = n;
-    p.kv_tiles[r] = (n + BN - 1) / BN;
-    p.q_tiles[r] = (n + BM - 1) / BM;
+    const int nk = a->k[r].n, nq = (r == RA_REF && !ref_rows) ? 0 : a->q[r].n;
+    p.nk[r] = nk;
+    p.nq[r] = nq;
+    p.kv_tiles[r] = (nk + BN - 1) / BN;
+    p.q_tiles[r] = (nq + BM - 1) / BM;
     p.q_blocks[r] = (p.q_tiles[r] + 1) / 2;
-    if (n == 0) continue;
-    if (!encode_seg(&p.tm_k[r], a->k[r], a->B, a->H, d, 64, BN, true) || !encode_seg(&p.tm_v[r], a->v[r], a->B, a->H, d, 64, BN, true))
+    if (nk > 0 && (!encode_seg(&p.tm_k[r], a->k[r], a->B, a->H, d, 64, BN, true) ||
+                   !encode_seg(&p.tm_v[r], a->v[r], a->B, a->H, d, 64, BN, true)))
       return RA_EINVAL;
-    if (r == RA_REF && !ref_rows) {
-      p.q_tiles[r] = 0;
-      p.q_blocks[r] = 0;
-      continue;
-    }
+    if (nq == 0) continue;
     if (!encode_seg(&p.tm_q[r], a->q[r], a->B, a->H, d, 64, BM, true)) return RA_EINVAL;
     p.o_ptr[r] = static_cast<__nv_bfloat16*>(a->o[r].ptr);
     p.o_sb[r] = a->o[r].stride_b;
     p.o_sh[r] = a->o[r].stride_h;
     p.o_sn[r] = a->o[r].stride_n;
   }
-  (void)n_ref;
   p.B = a->B;
   p.H = a->H;
   p.mass_rows = a->mass_rows;
-  p.mpl = refadapt_mass_partial_len(a->k[RA_TEXT].n, a->k[RA_TGT].n);
+  p.mpl = refadapt_mass_partial_len(a->q[RA_TEXT].n, a->q[RA_TGT].n);
   const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / std::sqrt(float(d));
   p.scale_log2 = scale * kLog2e;
   p.bias = a->ref_logit_bias;

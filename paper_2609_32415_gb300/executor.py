@@ -40,11 +40,21 @@ class Executor:
     query to its value at the block's last materialisation, App. A.2, times M;
     the executor keeps that anchor per block). The fixed-interval baseline is
     theta = inf with delta_max = the interval.
+
+    ``diagnostics`` adds, after every block, the staleness diagnostics of
+    Sec. 3.3 / App. A.2 on the target rows 0, k, 2k, ... (k =
+    ``diag_row_stride``), all through the same entry points: E_K, E_V (Eq. 7,
+    this step's reference K, V against the cache slot, refadapt_q_delta), a
+    second attention pass of the text and sampled target rows with the fresh
+    reference K/V (Eq. 8; its mass partials give the fresh exposure), and I_KV
+    (Eq. 10, refadapt_q_delta of the executed target output against it).
+    Logged per step in E_K, E_V, I_KV [steps, blocks, B, H] and M_fresh_part
+    [steps, blocks, B, H, tiles].
     """
 
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
                  mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
-                 device="cuda", cue="product"):
+                 device="cuda", cue="product", diagnostics=False, diag_row_stride=1):
         if cue not in CUES:
             raise ValueError("unknown cue %r" % (cue,))
         self.cue = cue
@@ -74,6 +84,20 @@ class Executor:
         self._prev_qtgt = [None] * n_blocks
         self.anchor = (torch.zeros((n_blocks, B, H, n_tgt, d), dtype=torch.bfloat16, device=dev)
                        if cue == "anchor_product" else None)
+        self.diagnostics = bool(diagnostics)
+        self.diag_row_stride = int(diag_row_stride)
+        if self.diagnostics:
+            k = self.diag_row_stride
+            n_s = (n_tgt + k - 1) // k
+            self.n_tgt_sampled = n_s
+            self.E_K = torch.zeros((self.log_steps, n_blocks, B, H), dtype=torch.float32, device=dev)
+            self.E_V = torch.zeros_like(self.E_K)
+            self.I_KV = torch.zeros_like(self.E_K)
+            self.mpl_fresh = api.refadapt_mass_partial_len(n_text, n_s)
+            self.M_fresh_part = torch.zeros((self.log_steps, n_blocks, B, H, self.mpl_fresh), dtype=torch.float32,
+                                            device=dev)
+            self._o_fresh = {"text": torch.empty((B, H, n_text, d), dtype=torch.bfloat16, device=dev),
+                             "tgt": torch.empty((B, H, n_s, d), dtype=torch.bfloat16, device=dev)}
         self._out = None
         self.attn_hook = None   # optional callable(phase in {"pre", "post"}, t, b), e.g. CUDA events
 
@@ -118,7 +142,22 @@ class Executor:
             mass_rows=self.mass_rows, err_word=self.err, stream=stream)
         if self.attn_hook is not None:
             self.attn_hook("post", t, b)
+        if self.diagnostics:
+            self._diagnose(t, b, li, x, out, stream)
         self._prev_qtgt[b] = qt
+
+    def _diagnose(self, t, b, li, x, out, stream):
+        k = self.diag_row_stride
+        qr, kr, vr = x["ref"]
+        api.refadapt_q_delta(kr, self.cache_k[b], self.E_K[li, b], self.workspace, self.eps, stream)
+        api.refadapt_q_delta(vr, self.cache_v[b], self.E_V[li, b], self.workspace, self.eps, stream)
+        q_s = x["tgt"][0][:, :, ::k, :]
+        api.refadapt_joint_attn(
+            (x["text"][0], None, q_s), (x["text"][1], kr, x["tgt"][1]), (x["text"][2], vr, x["tgt"][2]),
+            (self._o_fresh["text"], None, self._o_fresh["tgt"]), self.M_fresh_part[li, b],
+            softmax_scale=self.softmax_scale, ref_logit_bias=self.bias, err_word=self.err, stream=stream)
+        api.refadapt_q_delta(out["tgt"][:, :, ::k, :], self._o_fresh["tgt"], self.I_KV[li, b], self.workspace,
+                             self.eps, stream)
 
     def step(self, t, inputs, outs=None, log_index=None, stream=None, after_block=None):
         """Enqueue one denoising step. inputs[b]: dict role -> (q, k, v);

@@ -176,3 +176,29 @@ def test_attention_invalid_arguments(cuda_ok):
     with pytest.raises(RefAdaptError):
         api.refadapt_joint_attn([segs["text"][0], segs["ref"][0], mis], [segs[r][1] for r in ROLES],
                                 [segs[r][2] for r in ROLES], [out[r] for r in ROLES], mp)
+
+
+def test_attention_sampled_query_rows(cuda_ok):
+    """Query rows of a role may be a row sample (here every third target row,
+    a strided view) while every key row of the role is attended to."""
+    from paper_2609_32415_gb300 import api
+    n = dict(text=40, ref=260, tgt=301)
+    B, H, d = 2, 3, 128
+    segs = make_segments(B, H, d, n, gen=torch.Generator().manual_seed(14))
+    q_s = segs["tgt"][0][:, :, ::3, :]
+    ns = q_s.shape[2]
+    o = {"text": torch.full((B, H, 40, d), float("nan"), dtype=torch.bfloat16, device="cuda"),
+         "tgt": torch.full((B, H, ns, d), float("nan"), dtype=torch.bfloat16, device="cuda")}
+    mp = torch.zeros((B, H, api.refadapt_mass_partial_len(40, ns)), device="cuda")
+    api.refadapt_joint_attn([segs["text"][0], None, q_s], [segs[r][1] for r in ROLES], [segs[r][2] for r in ROLES],
+                            [o["text"], None, o["tgt"]], mp)
+    torch.cuda.synchronize()
+    sub = {r: list(segs[r]) for r in ROLES}
+    sub["tgt"][0] = q_s
+    for s in range(B):
+        ref = oracle_block(sub, s, REUSE, 1 / math.sqrt(d))
+        for r in ("text", "tgt"):
+            ok, worst, nw = o_close(o[r][s].double().cpu().numpy(), ref["O"][r])
+            assert ok, (r, worst, nw)
+        got_m = mp[s].double().sum(-1).cpu().numpy() / ns
+        assert np.abs(got_m - ref["M"]).max() <= M_ABS

@@ -12,12 +12,12 @@ pytestmark = pytest.mark.gpu
 ROLES = ("text", "ref", "tgt")
 
 
-def _run_both(wl, o_sample=None, cue="product"):
+def _run_both(wl, o_sample=None, cue="product", diagnostics=False, diag_row_stride=1):
     from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
     traj = synth.Trajectory(wl, device="cuda")
     ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max,
                   wl.eps, mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
-                  log_steps=wl.n_steps, cue=cue)
+                  log_steps=wl.n_steps, cue=cue, diagnostics=diagnostics, diag_row_stride=diag_row_stride)
     keep, outs, D = {}, {}, np.zeros((wl.n_steps, wl.n_blocks, wl.B, wl.H))
     for t in range(wl.n_steps):
         xs, os_ = [], []
@@ -49,7 +49,14 @@ def _run_both(wl, o_sample=None, cue="product"):
 
     rec = oracle.closed_loop(raw, wl.n_steps, wl.n_blocks, wl.B, theta=wl.theta, delta_max=wl.delta_max,
                              eps=wl.eps, bias=wl.bias, mass_rows=wl.mass_rows,
-                             forced_boundary=wl.forced_boundary, tie=tie, o_rows=o_sample, cue=cue)
+                             forced_boundary=wl.forced_boundary, tie=tie, o_rows=o_sample, cue=cue,
+                             diagnostics=diagnostics, diag_row_stride=diag_row_stride)
+    if diagnostics:
+        rows_s = ex.n_tgt_sampled
+        diag = {"E_K": ex.E_K.double().cpu().numpy(), "E_V": ex.E_V.double().cpu().numpy(),
+                "I_KV": ex.I_KV.double().cpu().numpy(),
+                "M_fresh": ex.M_fresh_part.double().sum(-1).cpu().numpy() / rows_s}
+        return modes, gbar, Mlog, D, outs, rec, diag
     return modes, gbar, Mlog, D, outs, rec
 
 
@@ -122,3 +129,25 @@ def test_closed_loop_ablation_cues(cuda_ok, cue, theta):
                                tgt_drift=[0.05, 0.1, 0.2, 0.3, 0.4], theta=theta, delta_max=4)
     res = _run_both(wl, cue=cue)
     _compare(wl, *res)
+
+
+def test_closed_loop_staleness_diagnostics(cuda_ok):
+    """Eqs. 7-10 through the executor's diagnostic pass (every second target row)
+    against the oracle's closed loop: E_K, E_V exact to the Q-change tolerance,
+    the fresh exposure to the mass tolerance, and I_KV within 5e-3 (both
+    outputs it compares are rounded to bf16 on the GPU)."""
+    from paper_2609_32415_gb300 import synth
+    wl = synth.custom_workload(2, 4, 128, 33, 300, 200, n_blocks=3, n_steps=4, ref_drift=0.2,
+                               tgt_drift=[0.05, 0.2, 0.4], theta=0.08, delta_max=100)
+    *res, diag = _run_both(wl, diagnostics=True, diag_row_stride=2)
+    _compare(wl, *res)
+    rec = res[-1]
+    for t in range(1, wl.n_steps):
+        for b in range(wl.n_blocks):
+            r = rec[t][b]
+            for key in ("E_K", "E_V"):
+                want, got = r[key], diag[key][t, b]
+                ok = np.where(want > 0, np.abs(got - want) / np.maximum(want, 1e-30) <= D_REL, got <= 1e-6)
+                assert ok.all(), (t, b, key, got, want)
+            assert np.abs(diag["M_fresh"][t, b] - r["M_fresh"]).max() <= M_ABS, (t, b)
+            assert np.abs(diag["I_KV"][t, b] - r["I_KV"]).max() <= 5e-3, (t, b, diag["I_KV"][t, b], r["I_KV"])

@@ -438,3 +438,42 @@ def test_anchor_moves_with_materialisation():
             qt = oracle.bf16_to_f64(traj[(t, b)]["tgt"][0])
             qp = oracle.bf16_to_f64(traj[(t - 1, b)]["tgt"][0])
             np.testing.assert_allclose(rec[t][b]["D"], oracle.q_change(qt, qp), atol=1e-15)
+
+
+# --------------------------------------------------------------------------- staleness diagnostics
+def test_diagnostics_vanish_without_reference_drift():
+    """Eqs. 7-10: with no reference drift the cache equals the fresh K/V, so the
+    endpoint drift and the local impact are zero and both exposures agree."""
+    traj = _tiny_inputs(ref_drift=0.0, seed=10)
+    rec = oracle.closed_loop(lambda t, b: traj[(t, b)], 3, 2, 2, theta=math.inf, delta_max=100,
+                             diagnostics=True)
+    for t in range(1, 3):
+        for b in range(2):
+            r = rec[t][b]
+            assert np.all(r["E_K"] == 0) and np.all(r["E_V"] == 0) and np.all(r["E_KV"] == 0)
+            np.testing.assert_allclose(r["I_KV"], 0.0, atol=1e-15)
+            np.testing.assert_allclose(r["M_fresh"], r["M_cached"], atol=1e-15)
+
+
+def test_diagnostics_match_their_definitions():
+    """Eq. 7 on K and V against the step-0 cache; Eqs. 8-10 written out with
+    fresh and anchor keys for every second target row."""
+    traj = _tiny_inputs(ref_drift=0.3, seed=11)
+    rec = oracle.closed_loop(lambda t, b: traj[(t, b)], 3, 1, 2, theta=math.inf, delta_max=100,
+                             diagnostics=True, diag_row_stride=2)
+    r = rec[2][0]
+    for s in range(2):
+        k0 = oracle.bf16_to_f64(traj[(0, 0)]["ref"][1])[s]
+        k2 = oracle.bf16_to_f64(traj[(2, 0)]["ref"][1])[s]
+        num = np.sqrt(((k2 - k0) ** 2).sum(axis=(1, 2)))
+        den = np.sqrt((k0 ** 2).sum(axis=(1, 2))) + 1e-6
+        np.testing.assert_allclose(r["E_K"][s], num / den, rtol=1e-13)
+        fresh = {"text": traj[(2, 0)]["text"], "tgt": traj[(2, 0)]["tgt"], "ref": traj[(2, 0)]["ref"]}
+        stale = {"text": traj[(2, 0)]["text"], "tgt": traj[(2, 0)]["tgt"], "ref": traj[(0, 0)]["ref"]}
+        of, _ = _plain_block(fresh, s, 1 / math.sqrt(8))
+        os_, _ = _plain_block(stale, s, 1 / math.sqrt(8))
+        rows = np.arange(3 + 10, 3 + 10 + 7)[::2]
+        a, b_ = os_[:, rows], of[:, rows]
+        want = np.sqrt(((a - b_) ** 2).sum(axis=(1, 2))) / (np.sqrt((b_ ** 2).sum(axis=(1, 2))) + 1e-6)
+        np.testing.assert_allclose(r["I_KV"][s], want, rtol=1e-12)
+        assert np.all(r["I_KV"][s] > 0)
