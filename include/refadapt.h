@@ -135,15 +135,22 @@ int32_t refadapt_mass_partial_len(int32_t n_text, int32_t n_tgt);
  * "Runtime cues"):
  *   D[b][h] = ||q_cur - q_prev||_F / (||q_prev||_F + eps)
  * over the segment's n rows x d columns. Bandwidth-bound: reads both tensors
- * once with 16-byte loads, fp32 per-thread sums, fp64 across threads and
- * blocks in a fixed order (deterministic).
+ * once through bulk copies into shared memory, fp32 per-thread sums, fp64
+ * across threads and blocks in a fixed order (deterministic).
+ *
+ * A slab (one sample and head) of at most 8 x 256 units of 12 KB per tensor
+ * (n <= 98304 rows at d = 128, 196608 at d = 64) is reduced by one
+ * thread-block cluster through distributed shared memory and leaves the
+ * workspace untouched; longer slabs take a multi-block path whose ticket
+ * counters and partial sums live in the workspace.
  *
  *  q_cur, q_prev    segments with equal n (>= 1); d in {64, 128}.
  *  d_out            device [B][H] fp32.
  *  workspace        device scratch of refadapt_q_delta_workspace_size(B, H)
  *                   bytes, 16-byte aligned, zero-filled once before its first
  *                   use; every call leaves it ready for the next. Calls that
- *                   share a workspace must be stream-ordered.
+ *                   share a workspace must be stream-ordered. Required (not
+ *                   NULL) whatever the slab length.
  */
 size_t refadapt_q_delta_workspace_size(int32_t B, int32_t H);
 ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
@@ -157,7 +164,8 @@ ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B,
  * pay cudaMalloc's implicit device synchronisation. The paper has no
  * counterpart; this is an interface convenience only.
  *
- * The scratch (ticket counters and per-block partial sums) lives in a
+ * The scratch that the long-slab path needs (ticket counters and per-block
+ * partial sums; slabs that fit one cluster use none) lives in a
  * file-scope static device array inside the library, sized for at most
  * RA_Q_DELTA_NOALLOC_MAX_BH (= B * H) slabs, about 193 KB; every GPU that loads
  * the library holds it until the process exits. Larger B * H returns RA_EINVAL

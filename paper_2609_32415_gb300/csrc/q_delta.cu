@@ -16,6 +16,14 @@
 // slab in unit order and stores one slot per (slab, CTA); the slab's last
 // contributor (ticket counter) adds the slots in CTA order and writes D, then
 // re-arms the counter. Every sum has a fixed order, so D is deterministic.
+//
+// Cluster path (used whenever a slab fits one thread-block cluster): one
+// cluster of up to 8 CTAs per (sample, head) slab, each CTA streaming its
+// share of the slab's units through a 4-stage ring; every CTA stores its pair
+// of sums into the cluster leader's shared memory (distributed shared memory)
+// and, after one cluster barrier, the leader adds them in rank order and writes
+// D. No global atomics, fences or workspace: the reduction tail is one
+// cluster barrier. The path above remains for slabs too long for one cluster.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -225,6 +233,160 @@ __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_consta
   }
 }
 
+// ---------------------------------------------------------------- cluster path
+constexpr int CL_MAX_CS = 8;            // CTAs per cluster (portable limit)
+constexpr int CL_CONSUMERS = 4;
+constexpr int CL_STAGES = CL_CONSUMERS;  // stage s belongs to consumer warp s
+constexpr int CL_THREADS = 32 * (CL_CONSUMERS + 1);
+constexpr int CL_MAX_UNITS = 256;        // units per CTA
+constexpr int CL_OFF_BAR = CL_STAGES * 2 * UNIT_BYTES;
+constexpr int CL_OFF_MISC = CL_OFF_BAR + 2 * CL_STAGES * 8;  // abort flag
+constexpr int CL_OFF_SUMS = CL_OFF_MISC + 16;                 // double2 per unit
+constexpr int CL_OFF_SLOTS = CL_OFF_SUMS + CL_MAX_UNITS * 16;  // leader: double2 per rank
+constexpr int CL_SMEM_BYTES = CL_OFF_SLOTS + CL_MAX_CS * 16;
+constexpr int CL_SMEM_ALLOC = CL_SMEM_BYTES + 1024;
+
+struct ClusterParams {
+  CUtensorMap tm_c, tm_p;
+  const char* base_c;
+  const char* base_p;
+  int64_t c_sb, c_sh, p_sb, p_sh;
+  int64_t slab_bytes;
+  int32_t bulk;
+  int32_t H, rows_per_unit, per_slab, cs;
+  float eps;
+  float* d_out;
+  uint64_t budget_ns;
+};
+
+__device__ __forceinline__ void cluster_sync_all() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(CL_THREADS) q_delta_cluster_kernel(const __grid_constant__ ClusterParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + CL_OFF_BAR);
+  uint64_t* empty = full + CL_STAGES;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + CL_OFF_MISC);
+  double* sums = reinterpret_cast<double*>(smem + CL_OFF_SUMS);
+  double* slots = reinterpret_cast<double*>(smem + CL_OFF_SLOTS);
+  uint32_t rank;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
+  const int h = blockIdx.y, b = blockIdx.z;
+  const int k0 = int(int64_t(rank) * p.per_slab / p.cs);
+  const int nu = int(int64_t(rank + 1) * p.per_slab / p.cs) - k0;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < CL_STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  // Every CTA of the cluster has started (its shared memory exists) before any
+  // remote store below; also orders the barrier initialisation.
+  cluster_sync_all();
+  const WaitCtl ctl{abort_flag, nullptr, p.budget_ns};
+
+  if (warp == CL_CONSUMERS) {
+    if (lane == 0) {
+      // ---------------------------------------------------------- producer
+      if (!p.bulk) {
+        tma_prefetch_desc(&p.tm_c);
+        tma_prefetch_desc(&p.tm_p);
+      }
+      int issued = 0;
+      for (int i = 0; i < nu; ++i) {
+        const int s = i % CL_STAGES;
+        if (i >= CL_STAGES && !mbar_wait(empty + s, ((i / CL_STAGES) - 1) & 1, ctl)) break;
+        const int k = k0 + i;
+        if (p.bulk) {
+          const int64_t off = int64_t(k) * UNIT_BYTES;
+          const int64_t rem = p.slab_bytes - off;
+          const uint32_t bytes = uint32_t(rem < UNIT_BYTES ? rem : UNIT_BYTES);
+          mbar_arrive_expect_tx(full + s, 2 * bytes);
+          bulk_load(smem + s * 2 * UNIT_BYTES, p.base_c + b * p.c_sb + h * p.c_sh + off, bytes, full + s);
+          bulk_load(smem + s * 2 * UNIT_BYTES + UNIT_BYTES, p.base_p + b * p.p_sb + h * p.p_sh + off, bytes,
+                    full + s);
+        } else {
+          mbar_arrive_expect_tx(full + s, 2 * UNIT_BYTES);
+          tma_load_4d(smem + s * 2 * UNIT_BYTES, &p.tm_c, full + s, 0, k * p.rows_per_unit, h, b);
+          tma_load_4d(smem + s * 2 * UNIT_BYTES + UNIT_BYTES, &p.tm_p, full + s, 0, k * p.rows_per_unit, h, b);
+        }
+        ++issued;
+      }
+      if (*abort_flag) {
+        for (int s = 0; s < CL_STAGES; ++s) {
+          const int n_s = (issued > s) ? (issued - s + CL_STAGES - 1) / CL_STAGES : 0;
+          if (n_s > 0) mbar_wait_drain(full + s, (n_s - 1) & 1, p.budget_ns);
+        }
+      }
+    }
+  } else {
+    // ------------------------------------------------------------ consumers
+    for (int i = warp; i < nu; i += CL_CONSUMERS) {
+      const int s = i % CL_STAGES;
+      if (!__all_sync(0xffffffffu, mbar_wait(full + s, (i / CL_STAGES) & 1, ctl))) break;
+      const uint4* vc = reinterpret_cast<const uint4*>(smem + s * 2 * UNIT_BYTES);
+      const uint4* vp = reinterpret_cast<const uint4*>(smem + s * 2 * UNIT_BYTES + UNIT_BYTES);
+      uint64_t sd = f2_pack(0.f, 0.f), sp = sd;
+      int nvec = UNIT_BYTES / 16;
+      if (p.bulk) {
+        const int64_t rem = p.slab_bytes - int64_t(k0 + i) * UNIT_BYTES;
+        if (rem < UNIT_BYTES) nvec = int(rem / 16);
+      }
+      if (nvec == UNIT_BYTES / 16) {
+#pragma unroll 8
+        for (int m = 0; m < UNIT_BYTES / 16 / 32; ++m) acc16(vc[lane + 32 * m], vp[lane + 32 * m], sd, sp);
+      } else {
+        for (int v = lane; v < nvec; v += 32) acc16(vc[v], vp[v], sd, sp);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(empty + s);
+      float a0, a1, b0, b1;
+      f2_unpack(sd, a0, a1);
+      f2_unpack(sp, b0, b1);
+      double dd = double(a0) + double(a1), dp = double(b0) + double(b1);
+#pragma unroll
+      for (int o = 16; o > 0; o >>= 1) {
+        dd += __shfl_xor_sync(0xffffffffu, dd, o);
+        dp += __shfl_xor_sync(0xffffffffu, dp, o);
+      }
+      if (lane == 0) {
+        sums[2 * i] = dd;
+        sums[2 * i + 1] = dp;
+      }
+    }
+    named_bar_sync(1, 32 * CL_CONSUMERS);
+    if (threadIdx.x == 0) {
+      // This CTA's share in unit order, stored into the leader's slot `rank`.
+      double td = 0.0, tp = 0.0;
+      for (int i = 0; i < nu; ++i) {
+        td += sums[2 * i];
+        tp += sums[2 * i + 1];
+      }
+      if (*abort_flag) td = NAN;
+      uint32_t remote;
+      asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(slots)), "r"(0));
+      asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank), "d"(td) : "memory");
+      asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank + 8), "d"(tp) : "memory");
+    }
+  }
+  // All remote stores are done and visible to the leader; no CTA exits while
+  // another may still write into its shared memory.
+  cluster_sync_all();
+  if (rank == 0 && threadIdx.x == 0) {
+    double td = 0.0, tp = 0.0;
+    for (int r = 0; r < p.cs; ++r) {
+      td += slots[2 * r];
+      tp += slots[2 * r + 1];
+    }
+    p.d_out[b * p.H + h] = float(sqrt(td) / (sqrt(tp) + double(p.eps)));
+  }
+}
+
 }  // namespace qd
 }  // namespace ra
 
@@ -269,6 +431,64 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
   }
   const int n = q_cur->n;
   const int bh = B * H;
+  {
+    // Cluster path: one cluster of up to 8 CTAs per slab.
+    const int rows_per_unit = qd::UNIT_BYTES / (2 * d);
+    const int per_slab = (n + rows_per_unit - 1) / rows_per_unit;
+    const int cs = per_slab < qd::CL_MAX_CS ? per_slab : qd::CL_MAX_CS;
+    if ((per_slab + cs - 1) / cs <= qd::CL_MAX_UNITS) {
+      qd::ClusterParams c;
+      std::memset(&c, 0, sizeof(c));
+      c.bulk = (q_cur->stride_n == d && q_prev->stride_n == d) ? 1 : 0;
+      c.base_c = static_cast<const char*>(q_cur->ptr);
+      c.base_p = static_cast<const char*>(q_prev->ptr);
+      c.c_sb = q_cur->stride_b * 2;
+      c.c_sh = q_cur->stride_h * 2;
+      c.p_sb = q_prev->stride_b * 2;
+      c.p_sh = q_prev->stride_h * 2;
+      c.slab_bytes = int64_t(n) * d * 2;
+      c.H = H;
+      c.rows_per_unit = rows_per_unit;
+      c.per_slab = per_slab;
+      c.cs = cs;
+      c.eps = eps;
+      c.d_out = d_out;
+      c.budget_ns = wait_budget_ns();
+      if (!c.bulk && (!encode_seg(&c.tm_c, *q_cur, B, H, d, d, rows_per_unit, false) ||
+                      !encode_seg(&c.tm_p, *q_prev, B, H, d, d, rows_per_unit, false)))
+        return RA_EINVAL;
+      static std::once_flag once_cl;
+      static cudaError_t attr_cl = cudaSuccess;
+      std::call_once(once_cl, [] {
+        attr_cl = cudaFuncSetAttribute(qd::q_delta_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       qd::CL_SMEM_ALLOC);
+      });
+      if (attr_cl != cudaSuccess) {
+        set_error("refadapt_q_delta: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_cl));
+        return RA_ECUDA;
+      }
+      cudaLaunchConfig_t cfg;
+      std::memset(&cfg, 0, sizeof(cfg));
+      cfg.gridDim = dim3(cs, H, B);
+      cfg.blockDim = dim3(qd::CL_THREADS, 1, 1);
+      cfg.dynamicSmemBytes = qd::CL_SMEM_ALLOC;
+      cfg.stream = static_cast<cudaStream_t>(stream);
+      cudaLaunchAttribute attr[1];
+      attr[0].id = cudaLaunchAttributeClusterDimension;
+      attr[0].val.clusterDim.x = cs;
+      attr[0].val.clusterDim.y = 1;
+      attr[0].val.clusterDim.z = 1;
+      cfg.attrs = attr;
+      cfg.numAttrs = 1;
+      const cudaError_t e = cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel, c);
+      if (e != cudaSuccess) {
+        set_error("refadapt_q_delta: cluster launch failed: %s", cudaGetErrorString(e));
+        cudaGetLastError();
+        return RA_ECUDA;
+      }
+      return launch_status("refadapt_q_delta");
+    }
+  }
   qd::Params p;
   p.H = H;
   p.rows_per_unit = qd::UNIT_BYTES / (2 * d);

@@ -21,8 +21,10 @@ def _d(q_cur, q_prev, eps=1e-6, ws=None):
 
 @pytest.mark.parametrize("B,H,n,d", [(1, 8, 256, 64), (2, 3, 1, 128), (1, 24, 4096, 128),
                                      (2, 4, 127, 128), (1, 2, 129, 64), (3, 5, 1000, 64),
-                                     (1, 24, 16380, 128)])
+                                     (1, 24, 16380, 128), (1, 1, 100000, 128), (2, 1, 200000, 64)])
 def test_q_delta_matches_oracle(cuda_ok, B, H, n, d):
+    """Slabs up to 98k rows (d = 128) take the cluster path; the two largest
+    shapes take the workspace path (slab split over many CTAs with tickets)."""
     g = torch.Generator().manual_seed(n + d)
     prev = (torch.randn((B, H, n, d), generator=g) / d ** 0.5).to(torch.bfloat16)
     cur = (prev.float() + 0.3 * torch.randn((B, H, n, d), generator=g) / d ** 0.5).to(torch.bfloat16)

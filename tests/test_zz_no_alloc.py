@@ -47,3 +47,21 @@ def test_noalloc_rejects_sizes_beyond_its_scratch(cuda_ok):
     with pytest.raises(RefAdaptError) as e:
         api.refadapt_q_delta_noalloc(x, x, out)
     assert e.value.status == RA_EINVAL
+
+
+def test_noalloc_long_slab_uses_the_static_scratch(cuda_ok):
+    """A slab too long for one cluster of CTAs goes through the path that needs
+    scratch (per-slab tickets and partial sums): the static array serves it."""
+    from paper_2609_32415_gb300 import api
+    B, H, d = 1, 2, 128
+    g = torch.Generator().manual_seed(22)
+    ws = api.q_delta_workspace(B, H)
+    for n in (100000, 120000):
+        cur, prev = _pair(g, B, H, n, d, 0.2)
+        want = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
+        got = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
+        api.refadapt_q_delta(cur, prev, want, ws, 1e-6)
+        api.refadapt_q_delta_noalloc(cur, prev, got, 1e-6)
+        torch.cuda.synchronize()
+        w, o = want.double().cpu().numpy(), got.double().cpu().numpy()
+        assert (np.abs(o - w) / np.abs(w)).max() <= D_REL, n
