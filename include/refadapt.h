@@ -138,11 +138,14 @@ int32_t refadapt_mass_partial_len(int32_t n_text, int32_t n_tgt);
  * once through bulk copies into shared memory, fp32 per-thread sums, fp64
  * across threads and blocks in a fixed order (deterministic).
  *
- * A slab (one sample and head) of at most 8 x 256 units of 12 KB per tensor
- * (n <= 98304 rows at d = 128, 196608 at d = 64) is reduced by one
- * thread-block cluster through distributed shared memory and leaves the
- * workspace untouched; longer slabs take a multi-block path whose ticket
- * counters and partial sums live in the workspace.
+ * Each slab (one sample and head) is reduced by one thread-block cluster of
+ * up to 8 CTAs through distributed shared memory, leaving the workspace
+ * untouched, when a slab has at most 8 x 256 units of 12 KB per tensor
+ * (n <= 98304 rows at d = 128, 196608 at d = 64), all B * H clusters fit on
+ * the GPU at once, and they fill at least 60 % of the SMs (or of the units,
+ * for tiny inputs). Otherwise a
+ * multi-block path spreads the units over all SMs; its ticket counters and
+ * partial sums live in the workspace.
  *
  *  q_cur, q_prev    segments with equal n (>= 1); d in {64, 128}.
  *  d_out            device [B][H] fp32.

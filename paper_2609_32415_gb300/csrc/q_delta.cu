@@ -17,13 +17,15 @@
 // contributor (ticket counter) adds the slots in CTA order and writes D, then
 // re-arms the counter. Every sum has a fixed order, so D is deterministic.
 //
-// Cluster path (used whenever a slab fits one thread-block cluster): one
+// Cluster path (used when the slabs fit clusters that fill the GPU): one
 // cluster of up to 8 CTAs per (sample, head) slab, each CTA streaming its
-// share of the slab's units through a 4-stage ring; every CTA stores its pair
-// of sums into the cluster leader's shared memory (distributed shared memory)
-// and, after one cluster barrier, the leader adds them in rank order and writes
-// D. No global atomics, fences or workspace: the reduction tail is one
-// cluster barrier. The path above remains for slabs too long for one cluster.
+// contiguous share of the slab's units through an 8-stage ring (one CTA per
+// SM) or a 4-stage ring (two per SM), whichever fills the SMs better; every
+// CTA stores its pair of sums into the cluster leader's shared memory
+// (distributed shared memory) and, after one cluster barrier, the leader adds
+// them in rank order and writes D. No global atomics, fences or workspace: the
+// reduction tail is one cluster barrier. The path above remains for slabs too
+// long for one cluster and for too few slabs to fill the GPU.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -234,17 +236,23 @@ __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_consta
 }
 
 // ---------------------------------------------------------------- cluster path
-constexpr int CL_MAX_CS = 8;            // CTAs per cluster (portable limit)
-constexpr int CL_CONSUMERS = 4;
-constexpr int CL_STAGES = CL_CONSUMERS;  // stage s belongs to consumer warp s
-constexpr int CL_THREADS = 32 * (CL_CONSUMERS + 1);
-constexpr int CL_MAX_UNITS = 256;        // units per CTA
-constexpr int CL_OFF_BAR = CL_STAGES * 2 * UNIT_BYTES;
-constexpr int CL_OFF_MISC = CL_OFF_BAR + 2 * CL_STAGES * 8;  // abort flag
-constexpr int CL_OFF_SUMS = CL_OFF_MISC + 16;                 // double2 per unit
-constexpr int CL_OFF_SLOTS = CL_OFF_SUMS + CL_MAX_UNITS * 16;  // leader: double2 per rank
-constexpr int CL_SMEM_BYTES = CL_OFF_SLOTS + CL_MAX_CS * 16;
-constexpr int CL_SMEM_ALLOC = CL_SMEM_BYTES + 1024;
+constexpr int CL_MAX_CS = 8;       // CTAs per cluster (portable limit)
+constexpr int CL_MAX_UNITS = 256;  // units per CTA
+
+// Shared-memory layout of a cluster CTA with S stages (stage s belongs to
+// consumer warp s; warp S is the producer).
+template <int S>
+struct ClLayout {
+  static constexpr int THREADS = 32 * (S + 1);
+  static constexpr int OFF_BAR = S * 2 * UNIT_BYTES;
+  static constexpr int OFF_MISC = OFF_BAR + 2 * S * 8;          // abort flag
+  static constexpr int OFF_SUMS = OFF_MISC + 16;                 // double2 per unit
+  static constexpr int OFF_SLOTS = OFF_SUMS + CL_MAX_UNITS * 16;  // leader: double2 per rank
+  static constexpr int BYTES = OFF_SLOTS + CL_MAX_CS * 16;
+  static constexpr int ALLOC = BYTES + 1024;
+};
+static_assert(ClLayout<8>::ALLOC <= 232448, "shared memory budget");
+static_assert(2 * ClLayout<4>::ALLOC <= 232448, "two 4-stage CTAs per SM");
 
 struct ClusterParams {
   CUtensorMap tm_c, tm_p;
@@ -263,14 +271,17 @@ __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-__global__ void __launch_bounds__(CL_THREADS) q_delta_cluster_kernel(const __grid_constant__ ClusterParams p) {
+template <int S>
+__global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(const __grid_constant__ ClusterParams p) {
+  using L = ClLayout<S>;
+  constexpr int CL_STAGES = S, CL_CONSUMERS = S;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
-  uint64_t* full = reinterpret_cast<uint64_t*>(smem + CL_OFF_BAR);
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
   uint64_t* empty = full + CL_STAGES;
-  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + CL_OFF_MISC);
-  double* sums = reinterpret_cast<double*>(smem + CL_OFF_SUMS);
-  double* slots = reinterpret_cast<double*>(smem + CL_OFF_SLOTS);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC);
+  double* sums = reinterpret_cast<double*>(smem + L::OFF_SUMS);
+  double* slots = reinterpret_cast<double*>(smem + L::OFF_SLOTS);
   uint32_t rank;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
   const int h = blockIdx.y, b = blockIdx.z;
@@ -387,6 +398,55 @@ __global__ void __launch_bounds__(CL_THREADS) q_delta_cluster_kernel(const __gri
   }
 }
 
+// Clusters of cs CTAs of the S-stage kernel that can be resident at once on
+// the current device (cached per device); -1 with the error set on failure.
+// Also raises the kernels' dynamic shared-memory limit once per device.
+int max_active_clusters(int S, int cs) {
+  static std::mutex mu;
+  static int cache[64][2][CL_MAX_CS + 1];
+  static bool ready[64] = {false};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    set_error("refadapt_q_delta: no usable current device");
+    return -1;
+  }
+  std::lock_guard<std::mutex> lk(mu);
+  if (!ready[dev]) {
+    cudaError_t e = cudaFuncSetAttribute(q_delta_cluster_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         ClLayout<8>::ALLOC);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(q_delta_cluster_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               ClLayout<4>::ALLOC);
+    for (int si = 0; si < 2 && e == cudaSuccess; ++si) {
+      for (int c = 1; c <= CL_MAX_CS && e == cudaSuccess; ++c) {
+        cudaLaunchConfig_t cfg;
+        std::memset(&cfg, 0, sizeof(cfg));
+        cfg.gridDim = dim3(c, 1, 1);
+        cfg.blockDim = dim3(si == 0 ? ClLayout<8>::THREADS : ClLayout<4>::THREADS, 1, 1);
+        cfg.dynamicSmemBytes = si == 0 ? ClLayout<8>::ALLOC : ClLayout<4>::ALLOC;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = c;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        e = si == 0 ? cudaOccupancyMaxActiveClusters(&n, q_delta_cluster_kernel<8>, &cfg)
+                    : cudaOccupancyMaxActiveClusters(&n, q_delta_cluster_kernel<4>, &cfg);
+        cache[dev][si][c] = n;
+      }
+    }
+    if (e != cudaSuccess) {
+      set_error("refadapt_q_delta: cluster occupancy query: %s", cudaGetErrorString(e));
+      cudaGetLastError();
+      return -1;
+    }
+    ready[dev] = true;
+  }
+  return cache[dev][S == 8 ? 0 : 1][cs];
+}
+
 }  // namespace qd
 }  // namespace ra
 
@@ -432,11 +492,35 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
   const int n = q_cur->n;
   const int bh = B * H;
   {
-    // Cluster path: one cluster of up to 8 CTAs per slab.
+    // Cluster path. Stages S = 8 (one CTA per SM, 192 KB in flight) or S = 4
+    // (two CTAs per SM); cluster size cs <= 8. Clusters live inside one GPC,
+    // so how many fit at once depends on the GPU's floorplan: the runtime's
+    // occupancy query says, and only configurations whose B * H clusters all
+    // run in one wave are candidates. Among those the one with the most bytes
+    // in flight (CTAs x stages) wins. Taken when it occupies at least 60 % of
+    // the CTAs the multi-block path would run (min(SMs, units)).
     const int rows_per_unit = qd::UNIT_BYTES / (2 * d);
     const int per_slab = (n + rows_per_unit - 1) / rows_per_unit;
-    const int cs = per_slab < qd::CL_MAX_CS ? per_slab : qd::CL_MAX_CS;
-    if ((per_slab + cs - 1) / cs <= qd::CL_MAX_UNITS) {
+    const int64_t sms = num_sms();
+    int best_s = 0, best_cs = 0;
+    int64_t best_score = 0;
+    for (int S : {8, 4}) {
+      for (int cs = 1; cs <= qd::CL_MAX_CS && cs <= per_slab; ++cs) {
+        if ((per_slab + cs - 1) / cs > qd::CL_MAX_UNITS) continue;
+        const int fit = qd::max_active_clusters(S, cs);
+        if (fit < 0) return RA_ECUDA;
+        if (bh > fit) continue;
+        const int64_t score = int64_t(bh) * cs * S;
+        if (score > best_score) {
+          best_score = score;
+          best_s = S;
+          best_cs = cs;
+        }
+      }
+    }
+    const int64_t units_all = int64_t(bh) * per_slab;
+    const int64_t ticket_ctas = units_all < sms ? units_all : sms;
+    if (best_s != 0 && double(bh) * best_cs >= 0.6 * double(ticket_ctas)) {
       qd::ClusterParams c;
       std::memset(&c, 0, sizeof(c));
       c.bulk = (q_cur->stride_n == d && q_prev->stride_n == d) ? 1 : 0;
@@ -450,37 +534,28 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
       c.H = H;
       c.rows_per_unit = rows_per_unit;
       c.per_slab = per_slab;
-      c.cs = cs;
+      c.cs = best_cs;
       c.eps = eps;
       c.d_out = d_out;
       c.budget_ns = wait_budget_ns();
       if (!c.bulk && (!encode_seg(&c.tm_c, *q_cur, B, H, d, d, rows_per_unit, false) ||
                       !encode_seg(&c.tm_p, *q_prev, B, H, d, d, rows_per_unit, false)))
         return RA_EINVAL;
-      static std::once_flag once_cl;
-      static cudaError_t attr_cl = cudaSuccess;
-      std::call_once(once_cl, [] {
-        attr_cl = cudaFuncSetAttribute(qd::q_delta_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       qd::CL_SMEM_ALLOC);
-      });
-      if (attr_cl != cudaSuccess) {
-        set_error("refadapt_q_delta: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_cl));
-        return RA_ECUDA;
-      }
       cudaLaunchConfig_t cfg;
       std::memset(&cfg, 0, sizeof(cfg));
-      cfg.gridDim = dim3(cs, H, B);
-      cfg.blockDim = dim3(qd::CL_THREADS, 1, 1);
-      cfg.dynamicSmemBytes = qd::CL_SMEM_ALLOC;
+      cfg.gridDim = dim3(best_cs, H, B);
+      cfg.blockDim = dim3(best_s == 8 ? qd::ClLayout<8>::THREADS : qd::ClLayout<4>::THREADS, 1, 1);
+      cfg.dynamicSmemBytes = best_s == 8 ? qd::ClLayout<8>::ALLOC : qd::ClLayout<4>::ALLOC;
       cfg.stream = static_cast<cudaStream_t>(stream);
       cudaLaunchAttribute attr[1];
       attr[0].id = cudaLaunchAttributeClusterDimension;
-      attr[0].val.clusterDim.x = cs;
+      attr[0].val.clusterDim.x = best_cs;
       attr[0].val.clusterDim.y = 1;
       attr[0].val.clusterDim.z = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 1;
-      const cudaError_t e = cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel, c);
+      const cudaError_t e = best_s == 8 ? cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel<8>, c)
+                                        : cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel<4>, c);
       if (e != cudaSuccess) {
         set_error("refadapt_q_delta: cluster launch failed: %s", cudaGetErrorString(e));
         cudaGetLastError();

@@ -21,10 +21,14 @@ def _d(q_cur, q_prev, eps=1e-6, ws=None):
 
 @pytest.mark.parametrize("B,H,n,d", [(1, 8, 256, 64), (2, 3, 1, 128), (1, 24, 4096, 128),
                                      (2, 4, 127, 128), (1, 2, 129, 64), (3, 5, 1000, 64),
-                                     (1, 24, 16380, 128), (1, 1, 100000, 128), (2, 1, 200000, 64)])
+                                     (1, 24, 16380, 128), (2, 20, 700, 128), (8, 25, 130, 64),
+                                     (1, 1, 100000, 128), (2, 1, 200000, 64), (1, 2, 20000, 128)])
 def test_q_delta_matches_oracle(cuda_ok, B, H, n, d):
-    """Slabs up to 98k rows (d = 128) take the cluster path; the two largest
-    shapes take the workspace path (slab split over many CTAs with tickets)."""
+    """On a 152-SM GB300: (1, 24, ...) runs clusters of 5 CTAs with 8
+    stages, (2, 20, ...) clusters of 3 with 8 stages, (8, 25, ...) single-CTA
+    clusters with 4 stages; the last three (slabs too long for a cluster, or
+    too few slabs to fill the GPU) take the workspace path with per-slab
+    tickets."""
     g = torch.Generator().manual_seed(n + d)
     prev = (torch.randn((B, H, n, d), generator=g) / d ** 0.5).to(torch.bfloat16)
     cur = (prev.float() + 0.3 * torch.randn((B, H, n, d), generator=g) / d ** 0.5).to(torch.bfloat16)
