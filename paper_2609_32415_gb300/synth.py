@@ -277,3 +277,92 @@ def sweep_points():
             for reuse in (0.0, 0.5, 0.9):
                 pts.append((total, frac, reuse))
     return pts
+
+
+# --------------------------------------------------------------------------- DiT block stack
+# Inputs of the DiT-block stack around the attention (dual-stream MMDiT block:
+# text rows use the text stream's weights, reference and target rows the image
+# stream's). Random numbers only:
+#
+# * stack input rows [B, n_role, C], C = H d: text and reference rows
+#   N(0, 1), the same at every step; target rows x_0 = N(0, 1),
+#   x_t = bf16(x_{t-1} + tgt_drift * N(0, 1)) (the sampler's latent moving);
+# * AdaLN modulation per (step, block, stream), six fp32 vectors [B, C]:
+#   shift, scale ~ 0.1 N(0, 1), gate ~ 0.3 + 0.05 N(0, 1) drawn once per
+#   (block, stream), plus mod_drift * N(0, 1) per step (the timestep
+#   embedding moving);
+# * weights per (block, stream): linear weights bf16 N(0, 1) / sqrt(fan_in),
+#   biases fp32 0.02 N(0, 1), q/k norm weights fp32 1 + 0.1 N(0, 1).
+MOD_NAMES = ("shift_a", "scale_a", "gate_a", "shift_m", "scale_m", "gate_m")
+STREAMS = ("text", "image")
+
+
+class DiTInputs:
+    """Seeded inputs of a DiT-block stack over a workload's row partition."""
+
+    def __init__(self, wl: Workload, device="cpu", mlp_ratio: int = 4, tgt_drift: float = 0.2,
+                 mod_drift: float = 0.05, weight_cache: bool = True):
+        self.wl = wl
+        self.device = torch.device(device)
+        self.C = wl.H * wl.d
+        self.F = mlp_ratio * self.C
+        self.tgt_drift = float(tgt_drift)
+        self.mod_drift = float(mod_drift)
+        self._x = None
+        self._w = {} if weight_cache else None
+
+    def _randn(self, shape, *parts):
+        g = _gen(self.device, self.wl.seed, 0xD17, *parts)
+        return torch.randn(shape, generator=g, device=self.device, dtype=torch.float32)
+
+    def h_in(self, t: int) -> Dict[str, torch.Tensor]:
+        """dict role -> bf16 [B, n_role, C] input rows of the stack at step t."""
+        wl = self.wl
+        out = {}
+        for r in ("text", "ref"):
+            out[r] = self._randn((wl.B, wl.n[r], self.C), 1, _ROLE_ID[r]).to(torch.bfloat16)
+        if self._x is None or self._x[0] > t:
+            self._x = (0, self._randn((wl.B, wl.n_tgt, self.C), 1, _ROLE_ID["tgt"]).to(torch.bfloat16))
+        cur, x = self._x
+        while cur < t:
+            cur += 1
+            x = (x.float() + self.tgt_drift * self._randn((wl.B, wl.n_tgt, self.C), 2, cur)).to(torch.bfloat16)
+        self._x = (cur, x)
+        out["tgt"] = x
+        return out
+
+    def mods(self, t: int, b: int) -> Dict[str, Dict[str, torch.Tensor]]:
+        """dict stream -> dict name -> fp32 [B, C] modulation vectors."""
+        wl = self.wl
+        out = {}
+        for si, st in enumerate(STREAMS):
+            d = {}
+            for j, name in enumerate(MOD_NAMES):
+                base = self._randn((wl.B, self.C), 3, b, si, j)
+                v = (0.3 + 0.05 * base) if name.startswith("gate") else 0.1 * base
+                if t > 0 and self.mod_drift > 0:
+                    v = v + self.mod_drift * self._randn((wl.B, self.C), 4, t, b, si, j)
+                d[name] = v.contiguous()
+            out[st] = d
+        return out
+
+    def weights(self, b: int) -> Dict[str, Dict[str, torch.Tensor]]:
+        """dict stream -> w_qkv [3C, C], w_o [C, C], w_1 [F, C], w_2 [C, F]
+        (bf16), b_qkv, b_o, b_1, b_2 (fp32), q_norm, k_norm [d] (fp32)."""
+        if self._w is not None and b in self._w:
+            return self._w[b]
+        C, F, d = self.C, self.F, self.wl.d
+        out = {}
+        for si, st in enumerate(STREAMS):
+            w = {}
+            for j, (name, shape, fan) in enumerate((("w_qkv", (3 * C, C), C), ("w_o", (C, C), C),
+                                                     ("w_1", (F, C), C), ("w_2", (C, F), F))):
+                w[name] = (self._randn(shape, 5, b, si, j) / math.sqrt(fan)).to(torch.bfloat16)
+            for j, (name, n) in enumerate((("b_qkv", 3 * C), ("b_o", C), ("b_1", F), ("b_2", C))):
+                w[name] = 0.02 * self._randn((n,), 6, b, si, j)
+            w["q_norm"] = 1.0 + 0.1 * self._randn((d,), 7, b, si, 0)
+            w["k_norm"] = 1.0 + 0.1 * self._randn((d,), 7, b, si, 1)
+            out[st] = w
+        if self._w is not None:
+            self._w[b] = out
+        return out
