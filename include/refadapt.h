@@ -270,6 +270,121 @@ ra_status refadapt_ref_cache_update(const ra_seg* k_src, const ra_seg* v_src, co
                                     int32_t x_width, const int32_t* mode, int32_t t, int32_t* a_b,
                                     void* stream);
 
+/* ------------------------------------------------------------------ DiT block around the attention
+ * The paper's models are DiTs whose blocks run joint attention over
+ * [text; reference; target] rows (Sec. 3, "Setting"). Under reuse the
+ * reference-side QKV projections and the other reference-stream operations
+ * are skipped because the layer-wise reference K/V are cached (App. A.4);
+ * at the boundary the cached reference hidden state is restored, its query
+ * runs against the current target and the reference output becomes the next
+ * block's cached hidden state (Algorithm 1, App. A.3). The paper does not
+ * give the block's layers; these entry points build a dual-stream MMDiT
+ * block (text rows with one weight set, reference and target rows with
+ * another) from: a modulated LayerNorm (refadapt_ln_modulate), linear layers
+ * with fused epilogues (refadapt_gemm) and the RoPE table the QKV epilogue
+ * reads (refadapt_rope_table).
+ *
+ * Rows come in up to three segments (text, reference, target), each with its
+ * own pointers and strides; row r of sample s of a segment lives at
+ * ptr + s * stride_s + r * stride_r (elements, features contiguous). A
+ * segment with gated = 1 is skipped for samples whose mode (device [B],
+ * written by refadapt_gate) is RA_MODE_REUSE. All calls are asynchronous on
+ * `stream` and allocate nothing; invalid arguments return RA_EINVAL before
+ * anything is launched.
+ */
+
+/* refadapt_rope_table — table[pos][i] = (cos, sin)(pos * base^(-2i/d)),
+ * fp32, pos in [0, n_pos), i in [0, d/2): [n_pos][d/2][2] floats, 16-byte
+ * aligned (device, caller-owned). Angles in fp64. d a multiple of 4. */
+ra_status refadapt_rope_table(float* table, int32_t n_pos, int32_t d, double base, void* stream);
+
+/* refadapt_ln_modulate — x = LN(h) * (1 + scale[s]) + shift[s] per row:
+ * LN without affine over C features, fp32 mean and variance, eps added to
+ * the variance; shift and scale are the block's AdaLN vectors for the row's
+ * stream and sample, fp32 [B][C] (row stride mod_stride_s). bf16 in and out;
+ * h and x must not overlap. C a multiple of 256, at most 4096; pointers
+ * 16-byte aligned, row strides >= C and multiples of 8 elements. */
+typedef struct {
+  const void* h;
+  int64_t h_stride_s, h_stride_r;
+  void* x;
+  int64_t x_stride_s, x_stride_r;
+  const float* shift;
+  const float* scale;
+  int64_t mod_stride_s;
+  int32_t rows;       /* rows per sample, >= 0 */
+  int32_t gated;
+} ra_lnmod_seg;
+
+typedef struct {
+  int32_t B, C, n_seg, reserved;
+  float eps, reserved2;
+  ra_lnmod_seg seg[3];
+  const int32_t* mode;  /* device [B]; required when a segment is gated */
+} ra_lnmod_args;
+
+ra_status refadapt_ln_modulate(const ra_lnmod_args* args, void* stream);
+
+/* refadapt_gemm — out = epilogue(A W^T + bias) on tcgen05 tensor cores:
+ * A bf16 rows of each segment (K features), W bf16 [N][K] (nn.Linear
+ * layout, one weight matrix per segment, so text and image streams differ),
+ * bias fp32 [N] or NULL, fp32 accumulation. N a multiple of 256, K of 64.
+ * Epilogues (fp32 until one final rounding to bf16):
+ *   RA_EPI_STORE  out = acc + bias
+ *   RA_EPI_GELU   out = gelu_tanh(acc + bias)
+ *   RA_EPI_RESID  out = resid + gate[s] * (acc + bias); gate fp32 [B][N]
+ *                 (row stride gate_stride_s); resid may equal out
+ *                 (in-place update of a residual stream) but must not
+ *                 partially overlap it.
+ *   RA_EPI_QKV    N = 3 H d, columns [q | k | v], head h at h*d within each
+ *                 part: q and k of each head are RMS-normalised over d
+ *                 (fp32, norm_eps added to the mean square) and scaled by
+ *                 q_norm / k_norm [d], then rotated by RoPE on interleaved
+ *                 pairs (2i, 2i+1) at position pos_offset + r, reading
+ *                 rope[pos][i] (refadapt_rope_table, rope_len rows); v gets
+ *                 the bias only. Written head-major to q_out, k_out, v_out
+ *                 (ra_seg, n = rows): for a gated segment (the reference
+ *                 rows) the K and V tiles are also skipped when the mode is
+ *                 RA_MODE_BOUNDARY (the block keeps its cached K/V), so k_out
+ *                 and v_out can point straight at the block's cache slot.
+ * Pointers 16-byte aligned; row strides multiples of 8 elements; out rows
+ * hold N columns (out_stride_r >= N); A rows K (a_stride_r >= K).
+ * err_word: device int32 or NULL; bit 0 set if a device wait timed out.
+ */
+typedef enum { RA_EPI_STORE = 0, RA_EPI_GELU = 1, RA_EPI_RESID = 2, RA_EPI_QKV = 3 } ra_epilogue;
+
+typedef struct {
+  const void* a;
+  int64_t a_stride_s, a_stride_r;
+  int32_t rows;        /* rows per sample, >= 0 */
+  int32_t gated;
+  const void* w;       /* bf16 [N][K] */
+  const float* bias;   /* [N] or NULL */
+  void* out;           /* STORE / GELU / RESID */
+  int64_t out_stride_s, out_stride_r;
+  const void* resid;   /* RESID */
+  int64_t resid_stride_s, resid_stride_r;
+  const float* gate;   /* RESID: [B][N] */
+  int64_t gate_stride_s;
+  ra_seg q_out, k_out, v_out;          /* QKV: [B, H, rows, d] */
+  const float* q_norm;                 /* QKV: [d] */
+  const float* k_norm;                 /* QKV: [d] */
+  int32_t pos_offset;                  /* QKV: RoPE position of row 0 */
+  int32_t reserved;
+} ra_gemm_seg;
+
+typedef struct {
+  int32_t B, N, K, epilogue;
+  int32_t H, d, n_seg, rope_len;       /* H, d, rope_len: QKV only */
+  ra_gemm_seg seg[3];
+  const int32_t* mode;                 /* device [B]; required when a segment is gated */
+  const float* rope;                   /* QKV: [rope_len][d/2][2] */
+  float norm_eps, reserved;
+  int32_t* err_word;
+} ra_gemm_args;
+
+ra_status refadapt_gemm(const ra_gemm_args* args, void* stream);
+
 /* ------------------------------------------------------------------ misc */
 const char* refadapt_status_string(ra_status s);
 const char* refadapt_last_error(void);

@@ -22,8 +22,10 @@ EXPORTED = (
     "refadapt_q_delta", "refadapt_state_size", "refadapt_state_init", "refadapt_gate",
     "refadapt_ref_cache_update", "refadapt_status_string", "refadapt_last_error",
     "refadapt_set_wait_budget_ns", "refadapt_check_error", "refadapt_version",
-    "refadapt_selftest_wait_timeout", "refadapt_q_delta_noalloc",
+    "refadapt_selftest_wait_timeout", "refadapt_q_delta_noalloc", "refadapt_rope_table",
+    "refadapt_ln_modulate", "refadapt_gemm",
 )
+RA_EPI_STORE, RA_EPI_GELU, RA_EPI_RESID, RA_EPI_QKV = 0, 1, 2, 3
 
 
 class RaSeg(ctypes.Structure):
@@ -46,6 +48,35 @@ class RaGateArgs(ctypes.Structure):
                 ("q_delta", c_void_p), ("mass_partial_prev", c_void_p),
                 ("state", c_void_p), ("mode_out", c_void_p), ("gbar_out", c_void_p),
                 ("m_out", c_void_p)]
+
+
+class RaLnmodSeg(ctypes.Structure):
+    _fields_ = [("h", c_void_p), ("h_stride_s", c_int64), ("h_stride_r", c_int64),
+                ("x", c_void_p), ("x_stride_s", c_int64), ("x_stride_r", c_int64),
+                ("shift", c_void_p), ("scale", c_void_p), ("mod_stride_s", c_int64),
+                ("rows", c_int32), ("gated", c_int32)]
+
+
+class RaLnmodArgs(ctypes.Structure):
+    _fields_ = [("B", c_int32), ("C", c_int32), ("n_seg", c_int32), ("reserved", c_int32),
+                ("eps", c_float), ("reserved2", c_float), ("seg", RaLnmodSeg * 3), ("mode", c_void_p)]
+
+
+class RaGemmSeg(ctypes.Structure):
+    _fields_ = [("a", c_void_p), ("a_stride_s", c_int64), ("a_stride_r", c_int64),
+                ("rows", c_int32), ("gated", c_int32), ("w", c_void_p), ("bias", c_void_p),
+                ("out", c_void_p), ("out_stride_s", c_int64), ("out_stride_r", c_int64),
+                ("resid", c_void_p), ("resid_stride_s", c_int64), ("resid_stride_r", c_int64),
+                ("gate", c_void_p), ("gate_stride_s", c_int64),
+                ("q_out", RaSeg), ("k_out", RaSeg), ("v_out", RaSeg),
+                ("q_norm", c_void_p), ("k_norm", c_void_p), ("pos_offset", c_int32), ("reserved", c_int32)]
+
+
+class RaGemmArgs(ctypes.Structure):
+    _fields_ = [("B", c_int32), ("N", c_int32), ("K", c_int32), ("epilogue", c_int32),
+                ("H", c_int32), ("d", c_int32), ("n_seg", c_int32), ("rope_len", c_int32),
+                ("seg", RaGemmSeg * 3), ("mode", c_void_p), ("rope", c_void_p),
+                ("norm_eps", c_float), ("reserved", c_float), ("err_word", c_void_p)]
 
 
 class RefAdaptError(RuntimeError):
@@ -103,6 +134,12 @@ def load():
     lib.refadapt_q_delta_noalloc.restype = c_int32
     lib.refadapt_q_delta_noalloc.argtypes = [POINTER(RaSeg), POINTER(RaSeg), c_int32, c_int32, c_int32, c_float,
                                              c_void_p, c_void_p]
+    lib.refadapt_rope_table.restype = c_int32
+    lib.refadapt_rope_table.argtypes = [c_void_p, c_int32, c_int32, c_double, c_void_p]
+    lib.refadapt_ln_modulate.restype = c_int32
+    lib.refadapt_ln_modulate.argtypes = [POINTER(RaLnmodArgs), c_void_p]
+    lib.refadapt_gemm.restype = c_int32
+    lib.refadapt_gemm.argtypes = [POINTER(RaGemmArgs), c_void_p]
     lib.refadapt_selftest_wait_timeout.restype = c_int32
     lib.refadapt_selftest_wait_timeout.argtypes = [c_void_p, c_uint64, c_void_p]
     _lib = lib

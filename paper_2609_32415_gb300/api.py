@@ -16,7 +16,7 @@ __all__ = ["seg", "refadapt_joint_attn", "refadapt_mass_partial_len", "refadapt_
            "refadapt_q_delta_workspace_size", "refadapt_q_delta_noalloc", "refadapt_state_size", "refadapt_state_init",
            "refadapt_gate", "refadapt_ref_cache_update", "refadapt_set_wait_budget_ns",
            "refadapt_check_error", "refadapt_version", "refadapt_selftest_wait_timeout", "q_delta_workspace", "new_state",
-           "alloc_mass_partial"]
+           "alloc_mass_partial", "refadapt_rope_table", "rope_table", "refadapt_ln_modulate", "refadapt_gemm"]
 
 
 def _ptr(t):
@@ -164,3 +164,89 @@ def refadapt_selftest_wait_timeout(err_word, budget_ns, stream=None):
 
 def refadapt_version() -> int:
     return int(_lib.load().refadapt_version())
+
+
+# --------------------------------------------------------------------------- DiT block around the attention
+def _rows(t, what):
+    """(ptr, stride_s, stride_r, rows) of a [B, rows, F] CUDA tensor with contiguous last axis."""
+    if t.dim() != 3 or not t.is_cuda or (t.shape[2] > 1 and t.stride(2) != 1):
+        raise ValueError("%s: expected a [B, rows, F] CUDA tensor with contiguous last axis, got %s"
+                         % (what, tuple(t.shape)))
+    return (t.data_ptr() if t.numel() > 0 else None), t.stride(0), t.stride(1), t.shape[1]
+
+
+def refadapt_rope_table(table, n_pos, d, base=10000.0, stream=None):
+    return check("refadapt_rope_table", _lib.load().refadapt_rope_table(
+        _ptr(table), int(n_pos), int(d), float(base), _stream(stream)))
+
+
+def rope_table(n_pos, d, base=10000.0, device="cuda", stream=None):
+    """[n_pos, d/2, 2] fp32 (cos, sin) table built by refadapt_rope_table."""
+    t = torch.empty((int(n_pos), int(d) // 2, 2), dtype=torch.float32, device=device)
+    refadapt_rope_table(t, n_pos, d, base, stream)
+    return t
+
+
+def refadapt_ln_modulate(segs, C, eps=1e-6, mode=None, stream=None):
+    """segs: up to three dicts with h, x ([B, rows, C] bf16), shift, scale
+    ([B, C] fp32) and optional gated (bool)."""
+    a = _lib.RaLnmodArgs()
+    B = None
+    for i, sd in enumerate(segs):
+        hp, hs, hr, rows = _rows(sd["h"], "h")
+        xp, xs, xr, xrows = _rows(sd["x"], "x")
+        if xrows != rows:
+            raise ValueError("h and x rows differ")
+        B = sd["h"].shape[0]
+        s = a.seg[i]
+        s.h, s.h_stride_s, s.h_stride_r = hp, hs, hr
+        s.x, s.x_stride_s, s.x_stride_r = xp, xs, xr
+        s.shift, s.scale = _ptr(sd["shift"]), _ptr(sd["scale"])
+        s.mod_stride_s = sd["shift"].stride(0)
+        if sd["scale"].stride(0) != s.mod_stride_s:
+            raise ValueError("shift and scale must share a row stride")
+        s.rows, s.gated = int(rows), int(bool(sd.get("gated", False)))
+    a.B, a.C, a.n_seg = int(B), int(C), len(segs)
+    a.eps = float(eps)
+    a.mode = _ptr(mode)
+    return check("refadapt_ln_modulate", _lib.load().refadapt_ln_modulate(ctypes.byref(a), _stream(stream)))
+
+
+def refadapt_gemm(segs, N, K, epilogue, mode=None, rope=None, H=0, d=0, norm_eps=1e-6, err_word=None,
+                  stream=None):
+    """segs: up to three dicts with a ([B, rows, K] bf16), w ([N, K] bf16),
+    optional bias ([N] fp32), gated; plus per epilogue out ([B, rows, N]),
+    resid and gate ([B, N] fp32) for RESID, or q, k, v ([B, H, rows, d]),
+    q_norm, k_norm ([d] fp32) and pos_offset for QKV."""
+    a = _lib.RaGemmArgs()
+    B = None
+    for i, sd in enumerate(segs):
+        ap, ass, asr, rows = _rows(sd["a"], "a")
+        B = sd["a"].shape[0]
+        s = a.seg[i]
+        s.a, s.a_stride_s, s.a_stride_r, s.rows = ap, ass, asr, int(rows)
+        s.gated = int(bool(sd.get("gated", False)))
+        w = sd["w"]
+        if tuple(w.shape) != (int(N), int(K)) or not w.is_contiguous() or w.dtype != torch.bfloat16:
+            raise ValueError("w: expected a contiguous [N, K] = [%d, %d] bf16 tensor, got %s"
+                             % (N, K, tuple(w.shape)))
+        s.w = _ptr(w)
+        s.bias = _ptr(sd.get("bias"))
+        if sd.get("out") is not None:
+            s.out, s.out_stride_s, s.out_stride_r, _ = _rows(sd["out"], "out")
+        if sd.get("resid") is not None:
+            s.resid, s.resid_stride_s, s.resid_stride_r, _ = _rows(sd["resid"], "resid")
+        if sd.get("gate") is not None:
+            s.gate, s.gate_stride_s = _ptr(sd["gate"]), sd["gate"].stride(0)
+        if epilogue == _lib.RA_EPI_QKV:
+            s.q_out, s.k_out, s.v_out = seg(sd["q"]), seg(sd["k"]), seg(sd["v"])
+            s.q_norm, s.k_norm = _ptr(sd["q_norm"]), _ptr(sd["k_norm"])
+            s.pos_offset = int(sd.get("pos_offset", 0))
+    a.B, a.N, a.K, a.epilogue = int(B), int(N), int(K), int(epilogue)
+    a.H, a.d, a.n_seg = int(H), int(d), len(segs)
+    a.rope_len = int(rope.shape[0]) if rope is not None else 0
+    a.mode = _ptr(mode)
+    a.rope = _ptr(rope)
+    a.norm_eps = float(norm_eps)
+    a.err_word = _ptr(err_word)
+    return check("refadapt_gemm", _lib.load().refadapt_gemm(ctypes.byref(a), _stream(stream)))
