@@ -128,7 +128,7 @@ def post_attention(h, o, mod, W, eps=1e-6):
 
 def dit_closed_loop(h_in, mods, weights, n_steps, n_blocks, B, H, d, *, theta, delta_max, eps=1e-6,
                     ln_eps=1e-6, rope_base=10000.0, mass_rows=0, forced_boundary=-1, tie=None,
-                    cue="product", nthreads=None):
+                    tie_band=1e-4, cue="product", nthreads=None):
     """Algorithm 1 over a stack of DiT blocks (the block of this module).
 
     h_in(t) -> dict role -> uint16 bf16 bits [B, n_role, C]: the stack's input
@@ -148,6 +148,9 @@ def dit_closed_loop(h_in, mods, weights, n_steps, n_blocks, B, H, d, *, theta, d
     Hbar[b], the cache takes K, V (a_b = t), all rows attend, the reference
     output is stored as Hbar[b+1]. D is Eq. 1 on the post-RoPE target query,
     M the executed attention's exposure, both recorded for the next step.
+
+    ``tie(t, b, s)`` and ``tie_band``: as in ``Gate.decide`` (a score within
+    the band of theta adopts the given decision).
 
     Returns records[t][b] = dict(mode, gbar, D, M, a_b) and per step
     outputs[t] = dict(text, tgt [B, n, C], hbar [n_blocks + 1][B] arrays or
@@ -185,7 +188,7 @@ def dit_closed_loop(h_in, mods, weights, n_steps, n_blocks, B, H, d, *, theta, d
                                       ln_eps, rope_base) for s in range(B)]
             q_tgt = np.stack([qkv["tgt"][s][0] for s in range(B)])
             D = q_change(q_tgt, prev_q[b], eps) if (t >= 1 and prev_q[b] is not None) else None
-            modes, gbars = gate.decide(t, b, D, prev_M[b], tie=tie)
+            modes, gbars = gate.decide(t, b, D, prev_M[b], tie=tie, tie_band=tie_band)
             M = np.zeros((B, H))
             for s in range(B):
                 mode = modes[s]

@@ -1,0 +1,138 @@
+"""Closed-loop parity of the DiT-block stack: Algorithm 1 run by DiTExecutor
+over the C ABI against oracle.dit.dit_closed_loop on the same seeded bf16
+inputs, weights and AdaLN vectors (modes, D, M, the stack's output rows and
+the reference hidden-state cache).
+
+Tolerances: every activation is re-rounded to bf16 after each layer on both
+sides, and a value the GPU forms in fp32 can land one bf16 step away from the
+oracle's; those single-step differences travel on through later layers and
+blocks. D is compared at 1e-3 relative (the 1e-4 of the attention-only path
+holds for D on identical inputs; here the target query itself carries such
+steps), the gate's ties are excused within 1e-3 of theta, M at the 1e-3
+absolute of the attention path. The output rows after a stack of blocks:
+each block adds the attention path's error (P rounded to bf16 before P V,
+about 1e-3 relative) and the single-step bf16 differences of its layers, and
+the residual stream carries them to the end, so the bound on a 4-block stack
+is 3e-2 of (|r| + rms(r)) per element (three times the one-attention bound)
+and 1e-2 normwise.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import BOUNDARY, COMPUTE, FULL, REUSE
+from oracle import dit
+from _helpers import M_ABS, bits, f64, o_close
+
+pytestmark = pytest.mark.gpu
+
+D_REL_DIT = 1e-3
+TIE_BAND_DIT = 1e-3
+ROWS_REL_DIT = 3e-2
+ROWS_NORMWISE_DIT = 1e-2
+
+
+def _setup(B=2, H=4, d=64, n_text=37, n_ref=256, n_tgt=200, n_blocks=4, n_steps=4, seed=0):
+    from paper_2609_32415_gb300 import synth
+    wl = synth.custom_workload(B, H, d, n_text, n_ref, n_tgt, n_blocks=n_blocks, n_steps=n_steps, seed=seed)
+    di = synth.DiTInputs(wl, device="cuda")
+    return wl, di
+
+
+def _run(wl, di, theta, delta_max, forced_boundary=-1, cue="product"):
+    from paper_2609_32415_gb300 import DiTExecutor
+    ex = DiTExecutor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, theta, delta_max,
+                     forced_boundary=forced_boundary, log_steps=wl.n_steps, cue=cue)
+    D = np.zeros((wl.n_steps, wl.n_blocks, wl.B, wl.H))
+    inputs, outs = {}, {}
+    for t in range(wl.n_steps):
+        inputs[t] = {r: x.clone() for r, x in di.h_in(t).items()}
+
+        def grab(tt, bb):
+            D[tt, bb] = ex.D[bb].double().cpu().numpy()
+
+        ex.step(t, inputs[t], di.mods, di.weights, after_block=grab)
+        torch.cuda.synchronize()
+        outs[t] = {"text": f64(ex.h["text"]), "tgt": f64(ex.h["tgt"]),
+                   "hbar": [f64(x) if x is not None else None for x in ex.hbar]}
+    ex.check()
+    modes = ex.modes.cpu().numpy()
+    gbar = ex.gbar.double().cpu().numpy()
+    M = ex.M.double().cpu().numpy()
+
+    def h_in(t):
+        return {r: bits(x) for r, x in inputs[t].items()}
+
+    def mods(t, b):
+        return {st: {k: v.cpu().numpy() for k, v in m.items()} for st, m in di.mods(t, b).items()}
+
+    def weights(b):
+        return {st: {k: (bits(v) if k.startswith("w_") else v.cpu().numpy()) for k, v in w.items()}
+                for st, w in di.weights(b).items()}
+
+    rec, ref_out = dit.dit_closed_loop(h_in, mods, weights, wl.n_steps, wl.n_blocks, wl.B, wl.H, wl.d,
+                                       theta=theta, delta_max=delta_max, forced_boundary=forced_boundary,
+                                       tie=lambda t, b, s: modes[t, b, s] == BOUNDARY, tie_band=TIE_BAND_DIT,
+                                       cue=cue)
+    return modes, gbar, M, D, outs, rec, ref_out
+
+
+def _compare(wl, modes, gbar, M, D, outs, rec, ref_out):
+    for t in range(wl.n_steps):
+        for b in range(wl.n_blocks):
+            r = rec[t][b]
+            assert list(modes[t, b]) == r["mode"], (t, b, modes[t, b], r["mode"])
+            if t >= 1:
+                rel = np.abs(D[t, b] - r["D"]) / np.abs(r["D"])
+                assert rel.max() <= D_REL_DIT, (t, b, rel.max())
+                np.testing.assert_allclose(gbar[t, b], r["gbar"], rtol=2e-3, atol=1e-6)
+            if t + 1 < wl.n_steps:
+                # M logged at step t+1 is the exposure of step t's executed attention
+                assert np.abs(M[t + 1, b] - r["M"]).max() <= M_ABS, (t, b)
+        for s in range(wl.B):
+            for role in ("text", "tgt"):
+                ok, worst, nw = o_close(outs[t][role][s][None], ref_out[t][role][s][None], ROWS_REL_DIT)
+                assert ok and nw <= ROWS_NORMWISE_DIT, (t, s, role, worst, nw)
+            for b in range(1, wl.n_blocks + 1):
+                want = ref_out[t]["hbar"][b][s]
+                if want is None:
+                    continue
+                ok, worst, nw = o_close(outs[t]["hbar"][b][s][None], want[None], ROWS_REL_DIT)
+                assert ok and nw <= ROWS_NORMWISE_DIT, (t, b, s, "hbar", worst, nw)
+
+
+def test_dit_stack_forced_boundary_schedule(cuda_ok):
+    """Forced boundary at block 2 and a full refresh every 3 steps: the
+    schedule FULL / [REUSE, REUSE, BOUNDARY, COMPUTE] / ... exercises every
+    mode, the restored hidden state at the boundary and the cache writes."""
+    wl, di = _setup()
+    res = _run(wl, di, float("inf"), 3, forced_boundary=2)
+    _compare(wl, *res)
+    modes = res[0]
+    assert list(modes[1, :, 0]) == [REUSE, REUSE, BOUNDARY, COMPUTE]
+    assert (modes[3] == FULL).all()
+
+
+def test_dit_stack_threshold_gate(cuda_ok):
+    """The score-driven gate (Eqs. 12-13) on the DiT stack: theta set
+    between the step-1 scores the oracle sees with every block reusing."""
+    wl, di = _setup(seed=3)
+    from paper_2609_32415_gb300 import synth  # noqa: F401
+
+    def bits_inputs(t):
+        return {r: bits(x) for r, x in di.h_in(t).items()}
+
+    def mods(t, b):
+        return {st: {k: v.cpu().numpy() for k, v in m.items()} for st, m in di.mods(t, b).items()}
+
+    def weights(b):
+        return {st: {k: (bits(v) if k.startswith("w_") else v.cpu().numpy()) for k, v in w.items()}
+                for st, w in di.weights(b).items()}
+
+    probe, _ = dit.dit_closed_loop(bits_inputs, mods, weights, 2, wl.n_blocks, wl.B, wl.H, wl.d,
+                                   theta=float("inf"), delta_max=10)
+    g1 = np.array([probe[1][b]["gbar"] for b in range(wl.n_blocks)])
+    theta = float(np.median(g1))
+    res = _run(wl, di, theta, 10)
+    _compare(wl, *res)
