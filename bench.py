@@ -59,6 +59,9 @@ def parse_args():
                          "fixed interval 3) on the workload; one JSON line per variant")
     ap.add_argument("--diagnostics", action="store_true",
                     help="also time the trajectory with the staleness diagnostics on (every 8th target row)")
+    ap.add_argument("--dit", action="store_true",
+                    help="time the DiT-block stack (QKV / output projection / MLP GEMMs, LayerNorms and the "
+                         "attention hot path) under Algorithm 1 on the workload's row partition; one JSON line")
     ap.add_argument("--blocks", type=int, default=0,
                     help="run only the first N blocks of the stack (small profiling cases)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file")
@@ -776,8 +779,187 @@ def main_ablation(args):
     torch.cuda.empty_cache()
 
 
+# ----------------------------------------------------------------------------- DiT-block stack
+def dit_gemm_flops(wl, C, F, name, modes):
+    """FLOPs of one named GEMM launch of a DiT block for the per-sample modes
+    (reference rows skipped on REUSE; only their query on BOUNDARY)."""
+    tot = 0
+    for m in modes:
+        m = int(m)
+        ref = 0 if m == 0 else wl.n_ref
+        if name == "qkv":
+            tot += 2 * (wl.n_text + wl.n_tgt) * C * 3 * C
+        elif name == "qkv_ref":
+            tot += 0 if m == 0 else 2 * wl.n_ref * C * (C if m == 1 else 3 * C)
+        elif name == "o_proj":
+            tot += 2 * (wl.n_text + wl.n_tgt + ref) * C * C
+        elif name in ("mlp1", "mlp2"):
+            tot += 2 * (wl.n_text + wl.n_tgt + ref) * C * F
+    return tot
+
+
+def dit_tables(wl, device):
+    """Pre-generated stack inputs, AdaLN vectors and weights (nothing is drawn
+    inside a timed region)."""
+    from paper_2609_32415_gb300 import synth
+    di = synth.DiTInputs(wl, device=device)
+    h_in = [{r: x.clone() for r, x in di.h_in(t).items()} for t in range(wl.n_steps)]
+    mods = {(t, b): di.mods(t, b) for t in range(wl.n_steps) for b in range(wl.n_blocks)}
+    weights = [di.weights(b) for b in range(wl.n_blocks)]
+    return di, h_in, mods, weights
+
+
+def time_dit(wl, tables, warmup, steps, theta, delta_max, timing=False, clocks=None):
+    import torch
+    from paper_2609_32415_gb300 import DiTExecutor
+    di, h_in, mods, weights = tables
+    ex = DiTExecutor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, theta, delta_max,
+                     log_steps=wl.n_steps)
+    T = wl.n_steps
+
+    def mods_fn(t, b):
+        return mods[(t, b)]
+
+    def w_fn(b):
+        return weights[b]
+
+    for i in range(warmup):
+        ex.step(i % T, h_in[i % T], mods_fn, w_fn)
+    torch.cuda.synchronize()
+    gemm_ev, attn_ev = [], []
+    if timing:
+        def ghook(phase, name, t, b):
+            if phase == "pre":
+                e = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                e[0].record()
+                gemm_ev.append((name, t, b, e))
+            else:
+                gemm_ev[-1][3][1].record()
+
+        def ahook(phase, t, b):
+            if phase == "pre":
+                e = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                e[0].record()
+                attn_ev.append((t, b, e))
+            else:
+                attn_ev[-1][2][1].record()
+        ex.gemm_hook, ex.attn_hook = ghook, ahook
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    torch.cuda.synchronize()
+    if clocks:
+        clocks.start()
+    ev[0].record()
+    for k in range(steps):
+        t = (warmup + k) % T
+        ex.step(t, h_in[t], mods_fn, w_fn)
+        ev[k + 1].record()
+    torch.cuda.synchronize()
+    clk = clocks.stop() if clocks else None
+    ex.gemm_hook = ex.attn_hook = None
+    ex.check()
+    modes = ex.modes.cpu().numpy()
+    res = {"total_ms": ev[0].elapsed_time(ev[-1]), "per_step_ms": [ev[k].elapsed_time(ev[k + 1]) for k in range(steps)],
+           "modes": modes, "gbar": ex.gbar.cpu().numpy(), "clocks": clk,
+           "steps_t": [(warmup + k) % T for k in range(steps)]}
+    if timing:
+        g_ms, g_fl = 0.0, 0
+        for name, t, b, (e0, e1) in gemm_ev:
+            g_ms += e0.elapsed_time(e1)
+            g_fl += dit_gemm_flops(wl, ex.C, ex.F, name, modes[t, b])
+        a_ms, a_fl = 0.0, 0
+        for t, b, (e0, e1) in attn_ev:
+            a_ms += e0.elapsed_time(e1)
+            a_fl += sum(attn_flops(wl, m) for m in modes[t, b])
+        res.update(gemm_ms=g_ms, gemm_flops=g_fl, gemm_launches=len(gemm_ev), attn_ms=a_ms, attn_flops=a_fl,
+                   attn_launches=len(attn_ev))
+    del ex
+    return res
+
+
+def calibrate_dit_theta(wl, tables):
+    """theta just above the largest step-1 score among the first half of the
+    stack (scores taken with every block reusing at step 1), so the first
+    half reuses at step 1 and the boundary falls in the second half."""
+    r = time_dit(wl, tables, 0, 2, float("inf"), max(2, wl.delta_max))
+    g = r["gbar"][1, :, 0]
+    half = max(1, wl.n_blocks // 2)
+    return float(max(g[:half])) * 1.0001, [round(float(x), 5) for x in g]
+
+
+def cublas_context_tflops(M, K, N, reps=20):
+    """torch.matmul (cuBLAS) on one GEMM shape of the stack, timed the same
+    way: context for the tcgen05 GEMM's rate."""
+    import torch
+    a = torch.randn((M, K), device="cuda").to(torch.bfloat16)
+    w = torch.randn((N, K), device="cuda").to(torch.bfloat16)
+    out = torch.empty((M, N), dtype=torch.bfloat16, device="cuda")
+    for _ in range(3):
+        torch.matmul(a, w.t(), out=out)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda._sleep(10_000_000)
+    e0.record()
+    for _ in range(reps):
+        torch.matmul(a, w.t(), out=out)
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / reps
+    del a, w, out
+    return 2.0 * M * N * K / ms / 1e9
+
+
+def main_dit(args):
+    import torch
+    import __graft_entry__ as ge
+    from paper_2609_32415_gb300 import synth
+    ge.build()
+    wl = synth.make_workload(args.config)
+    if args.blocks > 0:
+        wl.n_blocks = min(wl.n_blocks, args.blocks)
+    peaks = load_peaks()
+    tables = dit_tables(wl, "cuda")
+    torch.cuda.synchronize()
+    theta, g1 = calibrate_dit_theta(wl, tables)
+    clocks = Clocks(0)
+    main = time_dit(wl, tables, args.warmup, args.steps, theta, wl.delta_max, timing=True, clocks=clocks)
+    refresh = None if args.no_refresh_baseline else time_dit(wl, tables, args.warmup, args.steps, theta, 1)
+    C = wl.H * wl.d
+    ctx = cublas_context_tflops(wl.n_text + wl.n_ref + wl.n_tgt, C, 3 * C)
+    gt = main["gemm_flops"] / (main["gemm_ms"] * 1e-3) / 1e12
+    at = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
+    ms = main["total_ms"] / args.steps
+    line = {
+        "workload": "DiT-block stack: " + WORKLOAD_NAMES[args.config] + (
+            " (first %d blocks)" % wl.n_blocks if args.blocks > 0 else ""),
+        "block": "dual-stream MMDiT, C=%d, MLP 4C, random weights (%.1f GB)" % (
+            C, sum(v.numel() * v.element_size() for w in tables[3] for st in w.values() for v in st.values()) / 1e9),
+        "metric": "ms per denoising step of the DiT-block stack, vs always-refresh",
+        "value": round(ms, 3), "unit": "ms/step", "higher_is_better": False, "steps": args.steps,
+        "warmup": args.warmup, "dtype": "bf16", "data": "synthetic (seeded inputs, AdaLN vectors and weights)",
+        "theta": round(theta, 6), "theta_recipe": "just above the largest step-1 score of the first half of the stack",
+        "step1_scores_all_reuse": g1,
+        "per_step_ms": [round(x, 3) for x in main["per_step_ms"]],
+        "timed_trajectory_steps": main["steps_t"],
+        "modes_per_step": {str(t): [int(x) for x in main["modes"][t, :, 0]] for t in sorted(set(main["steps_t"]))},
+        "gemm_tflops": round(gt, 1), "gemm_frac_of_bf16_peak": round(gt / peaks["bf16_sustained"], 4),
+        "gemm_share_of_step": round(main["gemm_ms"] / main["total_ms"], 4),
+        "attn_tflops": round(at, 1), "attn_share_of_step": round(main["attn_ms"] / main["total_ms"], 4),
+        "same_shape_cublas_tflops": round(ctx, 1),
+        "peak": peaks["bf16_sustained"], "peak_kind": "%s, sustained bf16" % peaks["source"],
+        "clocks": main["clocks"],
+    }
+    if refresh is not None:
+        rms = refresh["total_ms"] / args.steps
+        line["always_refresh_ms_per_step"] = round(rms, 3)
+        line["speedup_vs_always_refresh"] = round(rms / ms, 3)
+    emit(line, args)
+
+
 def main():
     args = parse_args()
+    if args.dit:
+        main_dit(args)
+        return
     if args.ablation:
         main_ablation(args)
         return
