@@ -350,6 +350,10 @@ ra_status refadapt_ln_modulate(const ra_lnmod_args* args, void* stream);
  * Pointers 16-byte aligned; row strides multiples of 8 elements; out rows
  * hold N columns (out_stride_r >= N); A rows K (a_stride_r >= K).
  * err_word: device int32 or NULL; bit 0 set if a device wait timed out.
+ * tile_mode: 0 picks CTA pairs (a cluster of two SMs running one
+ * cta_group::2 MMA on a 256 x 256 tile, each SM staging half of the operands)
+ * when the call has at least a wave of such tiles, else one CTA per 128 x 256
+ * tile; 1 and 2 force either (results are the same; tests use both).
  */
 typedef enum { RA_EPI_STORE = 0, RA_EPI_GELU = 1, RA_EPI_RESID = 2, RA_EPI_QKV = 3 } ra_epilogue;
 
@@ -379,7 +383,8 @@ typedef struct {
   ra_gemm_seg seg[3];
   const int32_t* mode;                 /* device [B]; required when a segment is gated */
   const float* rope;                   /* QKV: [rope_len][d/2][2] */
-  float norm_eps, reserved;
+  float norm_eps;
+  int32_t tile_mode;                   /* 0 auto, 1 one CTA per 128 x 256 tile, 2 CTA pairs on 256 x 256 */
   int32_t* err_word;
 } ra_gemm_args;
 

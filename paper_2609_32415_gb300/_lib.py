@@ -76,7 +76,7 @@ class RaGemmArgs(ctypes.Structure):
     _fields_ = [("B", c_int32), ("N", c_int32), ("K", c_int32), ("epilogue", c_int32),
                 ("H", c_int32), ("d", c_int32), ("n_seg", c_int32), ("rope_len", c_int32),
                 ("seg", RaGemmSeg * 3), ("mode", c_void_p), ("rope", c_void_p),
-                ("norm_eps", c_float), ("reserved", c_float), ("err_word", c_void_p)]
+                ("norm_eps", c_float), ("tile_mode", c_int32), ("err_word", c_void_p)]
 
 
 class RefAdaptError(RuntimeError):

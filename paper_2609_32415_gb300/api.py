@@ -213,7 +213,7 @@ def refadapt_ln_modulate(segs, C, eps=1e-6, mode=None, stream=None):
 
 
 def refadapt_gemm(segs, N, K, epilogue, mode=None, rope=None, H=0, d=0, norm_eps=1e-6, err_word=None,
-                  stream=None):
+                  tile_mode=0, stream=None):
     """segs: up to three dicts with a ([B, rows, K] bf16), w ([N, K] bf16),
     optional bias ([N] fp32), gated; plus per epilogue out ([B, rows, N]),
     resid and gate ([B, N] fp32) for RESID, or q, k, v ([B, H, rows, d]),
@@ -248,5 +248,6 @@ def refadapt_gemm(segs, N, K, epilogue, mode=None, rope=None, H=0, d=0, norm_eps
     a.mode = _ptr(mode)
     a.rope = _ptr(rope)
     a.norm_eps = float(norm_eps)
+    a.tile_mode = int(tile_mode)
     a.err_word = _ptr(err_word)
     return check("refadapt_gemm", _lib.load().refadapt_gemm(ctypes.byref(a), _stream(stream)))

@@ -5,8 +5,9 @@
 //   D[r, n] = sum_k A[r, k] W[n, k]        (A rows of one segment and sample,
 //                                           W in nn.Linear layout [N][K])
 //
-// Persistent CTAs (one per SM), 128 x 256 output tiles, K in 64-column
-// steps. Tiles are numbered segment-major, then sample, then row tile, then
+// Two kernels: CTA pairs on 256 x 256 output tiles (gemm_pair_kernel, below,
+// used when a call has at least a wave of such tiles) and one CTA per SM on
+// 128 x 256 tiles (gemm_kernel), both persistent, K in 64-column steps. Tiles are numbered segment-major, then sample, then row tile, then
 // column tile (columns fastest, so the CTAs that run at once share A rows and
 // stream W through L2); CTA c takes tiles c, c + G, c + 2G, ...
 //   warp 0      TMA producer: per K step one 128 x 64 A box and one 256 x 64 W
@@ -59,6 +60,21 @@ constexpr int THREADS = 192;
 constexpr int TMEM_COLS = 512;
 static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 
+// CTA-pair kernel: 256 x 256 output tiles; each CTA stages its 128 rows of A
+// and its 128-column half of the W tile (32 KB per stage, 6 stages; a
+// seventh stage measured no faster).
+constexpr int P_TM = 256;
+constexpr int P_STAGES = 6;
+constexpr int P_A_BYTES = 128 * BK * 2;
+constexpr int P_B_BYTES = 128 * BK * 2;
+constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
+constexpr int P_OFF_BAR = P_STAGES * P_STAGE_BYTES;
+constexpr int P_NUM_BARS = 2 * P_STAGES + 2 + 2 + 1;
+constexpr int P_OFF_MISC = P_OFF_BAR + P_NUM_BARS * 8;
+constexpr int P_SMEM_BYTES = P_OFF_MISC + 16;
+constexpr int P_SMEM_ALLOC = P_SMEM_BYTES + 1024;
+static_assert(P_SMEM_ALLOC <= 232448, "shared memory budget");
+
 struct Seg {
   int64_t tile_begin;
   int32_t rows, m_tiles, gated, pos_offset;
@@ -92,6 +108,7 @@ struct Tile {
   bool live;
 };
 
+template <int TM>  // output rows per tile: 128 (one CTA) or 256 (a CTA pair)
 __device__ __forceinline__ Tile decode(const Params& p, int64_t t) {
   Tile r;
   int g = 0;
@@ -102,7 +119,7 @@ __device__ __forceinline__ Tile decode(const Params& p, int64_t t) {
   r.seg = g;
   r.s = int(local / per_sample);
   const int64_t rem = local - int64_t(r.s) * per_sample;
-  r.m0 = int(rem / p.n_tiles_n) * BM;
+  r.m0 = int(rem / p.n_tiles_n) * TM;
   r.n0 = int(rem % p.n_tiles_n) * BN;
   r.live = true;
   if (sg.gated) {
@@ -113,9 +130,12 @@ __device__ __forceinline__ Tile decode(const Params& p, int64_t t) {
   return r;
 }
 
+// GELU, tanh form, through the identity 0.5 x (1 + tanh(u)) = x / (1 + e^(-2u)),
+// u = sqrt(2/pi) (x + 0.044715 x^3): one exponential and one division instead
+// of tanhf (e^(-2u) overflowing to +inf for very negative x gives -0).
 __device__ __forceinline__ float gelu_tanh(float x) {
   const float u = 0.7978845608028654f * fmaf(0.044715f * x * x, x, x);
-  return 0.5f * x * (1.f + tanhf(u));
+  return __fdividef(x, 1.f + __expf(-2.f * u));
 }
 
 __device__ __forceinline__ void store32(__nv_bfloat16* dst, const float (&x)[32]) {
@@ -148,6 +168,87 @@ __device__ __forceinline__ void load_acc(uint32_t taddr, const float* bias, int 
     for (int i = 0; i < 32; ++i) x[i] = __uint_as_float(v[i]);
   }
 }
+
+// Epilogue of one output tile for the calling thread's row r (within the
+// segment's sample): 256 accumulator columns at TMEM address `base`.
+__device__ __forceinline__ void epilogue_tile(const Params& p, const Tile& tl, int r, uint32_t base) {
+  const Seg& sg = p.seg[tl.seg];
+  const bool valid = r < sg.rows;
+  if (p.epi == RA_EPI_QKV) {
+    const int part = tl.n0 / p.C;               // 0 q, 1 k, 2 v
+    const int h0 = (tl.n0 - part * p.C) / p.d;  // first head of the tile
+    const int pos = sg.pos_offset + r;
+    for (int hh = 0; hh < BN / p.d; ++hh) {
+      const int cb = hh * p.d;                  // tile column of the head
+      const int h = h0 + hh;
+      __nv_bfloat16* drow = sg.dst[part] + tl.s * sg.dst_sb[part] + h * sg.dst_sh[part] +
+                            int64_t(valid ? r : 0) * sg.dst_sn[part];
+      if (part == 2) {
+        for (int c0 = 0; c0 < p.d; c0 += 32) {
+          float x[32];
+          load_acc(base + cb + c0, sg.bias, tl.n0 + cb + c0, x);
+          if (valid) store32(drow + c0, x);
+        }
+        continue;
+      }
+      float ss = 0.f;
+      for (int c0 = 0; c0 < p.d; c0 += 32) {
+        float x[32];
+        load_acc(base + cb + c0, sg.bias, tl.n0 + cb + c0, x);
+#pragma unroll
+        for (int j = 0; j < 32; ++j) ss = fmaf(x[j], x[j], ss);
+      }
+      const float rstd = rsqrtf(ss / float(p.d) + p.norm_eps);
+      const float* w = sg.norm_w[part];
+      const float4* cs = p.rope + int64_t(valid ? pos : 0) * (p.d / 4);
+      for (int c0 = 0; c0 < p.d; c0 += 32) {
+        float x[32];
+        load_acc(base + cb + c0, sg.bias, tl.n0 + cb + c0, x);
+        const float4* w4 = reinterpret_cast<const float4*>(w + c0);
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 wv = __ldg(w4 + q);
+          const float4 rc = valid ? __ldg(cs + c0 / 4 + q) : make_float4(1.f, 0.f, 1.f, 0.f);
+          const float a0 = x[4 * q] * rstd * wv.x, a1 = x[4 * q + 1] * rstd * wv.y;
+          const float b0 = x[4 * q + 2] * rstd * wv.z, b1 = x[4 * q + 3] * rstd * wv.w;
+          x[4 * q] = a0 * rc.x - a1 * rc.y;
+          x[4 * q + 1] = a0 * rc.y + a1 * rc.x;
+          x[4 * q + 2] = b0 * rc.z - b1 * rc.w;
+          x[4 * q + 3] = b0 * rc.w + b1 * rc.z;
+        }
+        if (valid) store32(drow + c0, x);
+      }
+    }
+  } else {
+    const int64_t orow = int64_t(tl.s) * sg.out_ss + int64_t(valid ? r : 0) * sg.out_sr;
+    for (int c0 = 0; c0 < BN; c0 += 32) {
+      const int n = tl.n0 + c0;
+      float x[32];
+      load_acc(base + c0, sg.bias, n, x);
+      if (p.epi == RA_EPI_GELU) {
+#pragma unroll
+        for (int j = 0; j < 32; ++j) x[j] = gelu_tanh(x[j]);
+      } else if (p.epi == RA_EPI_RESID && valid) {
+        const uint4* rp = reinterpret_cast<const uint4*>(sg.resid + int64_t(tl.s) * sg.res_ss +
+                                                         int64_t(r) * sg.res_sr + n);
+        const float4* gp = reinterpret_cast<const float4*>(sg.gate + int64_t(tl.s) * sg.gate_ss + n);
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const uint4 rv = rp[q];
+          const uint32_t w4[4] = {rv.x, rv.y, rv.z, rv.w};
+          const float4 g0 = __ldg(gp + 2 * q), g1 = __ldg(gp + 2 * q + 1);
+          const float gv[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float lo = __uint_as_float(w4[e] << 16), hi = __uint_as_float(w4[e] & 0xFFFF0000u);
+            x[8 * q + 2 * e] = fmaf(gv[2 * e], x[8 * q + 2 * e], lo);
+            x[8 * q + 2 * e + 1] = fmaf(gv[2 * e + 1], x[8 * q + 2 * e + 1], hi);
+          }
+        }
+      }
+      if (valid) store32(sg.out + orow + n, x);
+    }
+  }}
 
 __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant__ Params p) {
   extern __shared__ uint8_t smem_raw[];
@@ -192,7 +293,7 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
       int64_t it = 0;  // K steps issued
       bool ok = true;
       for (int64_t t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
-        const Tile tl = decode(p, t);
+        const Tile tl = decode<BM>(p, t);
         if (!tl.live) continue;
         for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
           const int st = int(it % STAGES);
@@ -219,7 +320,7 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
       int i = 0;
       bool ok = true, issued = false;
       for (int64_t t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
-        const Tile tl = decode(p, t);
+        const Tile tl = decode<BM>(p, t);
         if (!tl.live) continue;
         const int buf = i & 1, use = i >> 1;
         if (use > 0 && !(ok = mbar_wait(tempty + buf, uint32_t((use - 1) & 1), ctl))) break;
@@ -253,90 +354,12 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
     const uint32_t lane_off = uint32_t(quarter * 32) << 16;
     int i = 0;
     for (int64_t t = blockIdx.x; t < p.total_tiles; t += gridDim.x) {
-      const Tile tl = decode(p, t);
+      const Tile tl = decode<BM>(p, t);
       if (!tl.live) continue;
       const int buf = i & 1, use = i >> 1;
       if (!__all_sync(0xffffffffu, mbar_wait(tfull + buf, uint32_t(use & 1), ctl))) break;
       tc_fence_after();
-      const Seg& sg = p.seg[tl.seg];
-      const int r = tl.m0 + row;
-      const bool valid = r < sg.rows;
-      const uint32_t base = tmem + lane_off + uint32_t(buf * BN);
-      if (p.epi == RA_EPI_QKV) {
-        const int part = tl.n0 / p.C;               // 0 q, 1 k, 2 v
-        const int h0 = (tl.n0 - part * p.C) / p.d;  // first head of the tile
-        const int pos = sg.pos_offset + r;
-        for (int hh = 0; hh < BN / p.d; ++hh) {
-          const int cb = hh * p.d;                  // tile column of the head
-          const int h = h0 + hh;
-          __nv_bfloat16* drow = sg.dst[part] + tl.s * sg.dst_sb[part] + h * sg.dst_sh[part] +
-                                int64_t(valid ? r : 0) * sg.dst_sn[part];
-          if (part == 2) {
-            for (int c0 = 0; c0 < p.d; c0 += 32) {
-              float x[32];
-              load_acc(base + cb + c0, sg.bias, tl.n0 + cb + c0, x);
-              if (valid) store32(drow + c0, x);
-            }
-            continue;
-          }
-          float ss = 0.f;
-          for (int c0 = 0; c0 < p.d; c0 += 32) {
-            float x[32];
-            load_acc(base + cb + c0, sg.bias, tl.n0 + cb + c0, x);
-#pragma unroll
-            for (int j = 0; j < 32; ++j) ss = fmaf(x[j], x[j], ss);
-          }
-          const float rstd = rsqrtf(ss / float(p.d) + p.norm_eps);
-          const float* w = sg.norm_w[part];
-          const float4* cs = p.rope + int64_t(valid ? pos : 0) * (p.d / 4);
-          for (int c0 = 0; c0 < p.d; c0 += 32) {
-            float x[32];
-            load_acc(base + cb + c0, sg.bias, tl.n0 + cb + c0, x);
-            const float4* w4 = reinterpret_cast<const float4*>(w + c0);
-#pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const float4 wv = __ldg(w4 + q);
-              const float4 rc = valid ? __ldg(cs + c0 / 4 + q) : make_float4(1.f, 0.f, 1.f, 0.f);
-              const float a0 = x[4 * q] * rstd * wv.x, a1 = x[4 * q + 1] * rstd * wv.y;
-              const float b0 = x[4 * q + 2] * rstd * wv.z, b1 = x[4 * q + 3] * rstd * wv.w;
-              x[4 * q] = a0 * rc.x - a1 * rc.y;
-              x[4 * q + 1] = a0 * rc.y + a1 * rc.x;
-              x[4 * q + 2] = b0 * rc.z - b1 * rc.w;
-              x[4 * q + 3] = b0 * rc.w + b1 * rc.z;
-            }
-            if (valid) store32(drow + c0, x);
-          }
-        }
-      } else {
-        const int64_t orow = int64_t(tl.s) * sg.out_ss + int64_t(valid ? r : 0) * sg.out_sr;
-        for (int c0 = 0; c0 < BN; c0 += 32) {
-          const int n = tl.n0 + c0;
-          float x[32];
-          load_acc(base + c0, sg.bias, n, x);
-          if (p.epi == RA_EPI_GELU) {
-#pragma unroll
-            for (int j = 0; j < 32; ++j) x[j] = gelu_tanh(x[j]);
-          } else if (p.epi == RA_EPI_RESID && valid) {
-            const uint4* rp = reinterpret_cast<const uint4*>(sg.resid + int64_t(tl.s) * sg.res_ss +
-                                                             int64_t(r) * sg.res_sr + n);
-            const float4* gp = reinterpret_cast<const float4*>(sg.gate + int64_t(tl.s) * sg.gate_ss + n);
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const uint4 rv = rp[q];
-              const uint32_t w4[4] = {rv.x, rv.y, rv.z, rv.w};
-              const float4 g0 = __ldg(gp + 2 * q), g1 = __ldg(gp + 2 * q + 1);
-              const float gv[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const float lo = __uint_as_float(w4[e] << 16), hi = __uint_as_float(w4[e] & 0xFFFF0000u);
-                x[8 * q + 2 * e] = fmaf(gv[2 * e], x[8 * q + 2 * e], lo);
-                x[8 * q + 2 * e + 1] = fmaf(gv[2 * e + 1], x[8 * q + 2 * e + 1], hi);
-              }
-            }
-          }
-          if (valid) store32(sg.out + orow + n, x);
-        }
-      }
+      epilogue_tile(p, tl, tl.m0 + row, tmem + lane_off + uint32_t(buf * BN));
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(tempty + buf);
@@ -349,6 +372,157 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
     tc_fence_after();
     tmem_dealloc(tmem, TMEM_COLS);
   }
+}
+
+
+// CTA-pair variant (cluster of two, cta_group::2). Both CTAs walk the same
+// tile sequence (cluster c takes tiles c, c + G/2, ...); per K step each CTA's
+// producer loads its own 128 A rows and its half of the W tile, and both
+// loads complete on rank 0's full barrier (rank 0 arms it for both CTAs'
+// bytes). Rank 0's MMA thread issues M = 256, N = 256 MMAs; commits are
+// multicast to both CTAs (stage free, accumulator ready). Each CTA's epilogue
+// reads its own TMEM rows and arrives on rank 0's accumulator-free barrier
+// (count 8). The two CTAs meet at a cluster barrier before TMEM is freed and
+// before either exits, so no remote arrive or MMA outlives its target.
+__global__ void __launch_bounds__(THREADS, 1) gemm_pair_kernel(const __grid_constant__ Params p) {
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
+  uint64_t* bars = reinterpret_cast<uint64_t*>(smem + P_OFF_BAR);
+  uint64_t* full = bars;
+  uint64_t* empty = bars + P_STAGES;
+  uint64_t* tfull = bars + 2 * P_STAGES;
+  uint64_t* tempty = bars + 2 * P_STAGES + 2;
+  uint64_t* drain = bars + 2 * P_STAGES + 4;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + P_OFF_MISC);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + P_OFF_MISC + 4);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_rank();
+  const int64_t cid = blockIdx.x >> 1, ncl = gridDim.x >> 1;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < P_STAGES; ++s) {
+      mbar_init(full + s, 1);
+      mbar_init(empty + s, 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(tfull + b, 1);
+      mbar_init(tempty + b, 8);
+    }
+    mbar_init(drain, 1);
+    *abort_flag = 0;
+    fence_mbar_init();
+  }
+  if (warp == 1) tmem_alloc_pair(tmem_slot, TMEM_COLS);
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();  // both CTAs' barriers and TMEM exist before any cross-CTA use
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+  const WaitCtl ctl{abort_flag, p.err_word, p.budget_ns};
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // -------------------------------------------------------------- producer (both CTAs)
+      for (int g = 0; g < p.n_seg; ++g)
+        if (p.seg[g].rows > 0) {
+          tma_prefetch_desc(&p.tm_a[g]);
+          tma_prefetch_desc(&p.tm_w[g]);
+        }
+      const uint32_t full0 = mapa_shared(smem_u32(full), 0);  // rank 0's full barriers
+      int64_t it = 0;
+      bool ok = true;
+      for (int64_t t = cid; ok && t < p.total_tiles; t += ncl) {
+        const Tile tl = decode<P_TM>(p, t);
+        if (!tl.live) continue;
+        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+          const int st = int(it % P_STAGES);
+          if (it >= P_STAGES && !(ok = mbar_wait(empty + st, uint32_t((it / P_STAGES - 1) & 1), ctl))) break;
+          uint8_t* sa = smem + st * P_STAGE_BYTES;
+          if (rank == 0) mbar_arrive_expect_tx(full + st, 2 * P_STAGE_BYTES);
+          tma_load_4d_pair(sa, &p.tm_a[tl.seg], full0 + 8u * st, kb * BK, tl.m0 + int(rank) * 128, 0, tl.s);
+          tma_load_4d_pair(sa + P_A_BYTES, &p.tm_w[tl.seg], full0 + 8u * st, kb * BK, tl.n0 + int(rank) * 128, 0, 0);
+        }
+      }
+      if (*abort_flag) {
+        if (rank == 0) {
+          // rank 0's full barriers count both CTAs' bytes of every phase it armed
+          for (int st = 0; st < P_STAGES; ++st) {
+            const int64_t n_s = (it > st) ? (it - st + P_STAGES - 1) / P_STAGES : 0;
+            if (n_s > 0) mbar_wait_drain(full + st, uint32_t((n_s - 1) & 1), p.budget_ns);
+          }
+        } else {
+          // this CTA cannot observe its own loads' completion: give them time to land
+          const uint64_t t0 = globaltimer_ns();
+          while (globaltimer_ns() - t0 < 200000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // -------------------------------------------------------------- MMA issuer (rank 0)
+      constexpr uint32_t IDESC = idesc_bf16_f32(P_TM, BN, 0, 0);
+      const uint32_t s0 = smem_u32(smem);
+      int64_t it = 0;
+      int i = 0;
+      bool ok = true, issued = false;
+      for (int64_t t = cid; ok && t < p.total_tiles; t += ncl) {
+        const Tile tl = decode<P_TM>(p, t);
+        if (!tl.live) continue;
+        const int buf = i & 1, use = i >> 1;
+        if (use > 0 && !(ok = mbar_wait_cluster(tempty + buf, uint32_t((use - 1) & 1), ctl))) break;
+        tc_fence_after();
+        const uint32_t d_t = tmem + uint32_t(buf * BN);
+        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+          const int st = int(it % P_STAGES);
+          if (!(ok = mbar_wait(full + st, uint32_t((it / P_STAGES) & 1), ctl))) break;
+          tc_fence_after();
+          const uint32_t sa = s0 + st * P_STAGE_BYTES, sb = sa + P_A_BYTES;
+#pragma unroll
+          for (int kk = 0; kk < BK / 16; ++kk)
+            umma_ss_pair(d_t, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024), IDESC,
+                         (kb > 0 || kk > 0) ? 1u : 0u);
+          umma_commit_pair(empty + st, 0x3);
+          issued = true;
+        }
+        if (!ok) break;
+        umma_commit_pair(tfull + buf, 0x3);
+        ++i;
+      }
+      if (!ok && issued) {
+        umma_commit_pair(drain, 0x1);
+        mbar_wait_drain(drain, 0, p.budget_ns);
+      }
+    }
+  } else {
+    // ---------------------------------------------------------------- epilogue (both CTAs)
+    const int quarter = warp & 3;
+    const int row = int(rank) * 128 + quarter * 32 + lane;
+    const uint32_t lane_off = uint32_t(quarter * 32) << 16;
+    const uint32_t tempty0 = mapa_shared(smem_u32(tempty), 0);
+    int i = 0;
+    for (int64_t t = cid; t < p.total_tiles; t += ncl) {
+      const Tile tl = decode<P_TM>(p, t);
+      if (!tl.live) continue;
+      const int buf = i & 1, use = i >> 1;
+      if (!__all_sync(0xffffffffu, mbar_wait(tfull + buf, uint32_t(use & 1), ctl))) break;
+      tc_fence_after();
+      epilogue_tile(p, tl, tl.m0 + row, tmem + lane_off + uint32_t(buf * BN));
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (rank == 0)
+          mbar_arrive(tempty + buf);
+        else
+          mbar_arrive_remote(tempty0 + 8u * buf);
+      }
+      ++i;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync_all();
+  tc_fence_after();
+  if (warp == 1) tmem_dealloc_pair(tmem, TMEM_COLS);
 }
 
 __global__ void rope_table_kernel(float* table, int32_t n_pos, int32_t d, double base) {
@@ -427,6 +601,18 @@ extern "C" ra_status refadapt_gemm(const ra_gemm_args* a, void* stream) {
     p.rope = reinterpret_cast<const float4*>(a->rope);
     p.rope_len = a->rope_len;
   }
+  if (a->tile_mode < 0 || a->tile_mode > 2) {
+    set_error("refadapt_gemm: tile_mode %d (0 auto, 1 one CTA per tile, 2 CTA pairs)", a->tile_mode);
+    return RA_EINVAL;
+  }
+  // One CTA per 128-row tile, or CTA pairs on 256-row tiles when there is a
+  // full wave of pair tiles (auto) or when asked.
+  int64_t pair_tiles = 0;
+  for (int g = 0; g < a->n_seg; ++g)
+    if (a->seg[g].rows > 0) pair_tiles += int64_t(a->B) * ((a->seg[g].rows + P_TM - 1) / P_TM) * p.n_tiles_n;
+  const int sms = num_sms();
+  const bool pair = a->tile_mode == 2 || (a->tile_mode == 0 && sms >= 2 && pair_tiles >= sms / 2);
+  const int tm = pair ? P_TM : BM;
   int64_t tiles = 0;
   for (int g = 0; g < a->n_seg; ++g) {
     const ra_gemm_seg& s = a->seg[g];
@@ -437,7 +623,7 @@ extern "C" ra_status refadapt_gemm(const ra_gemm_args* a, void* stream) {
     }
     d.tile_begin = tiles;
     d.rows = s.rows;
-    d.m_tiles = (s.rows + BM - 1) / BM;
+    d.m_tiles = (s.rows + tm - 1) / tm;
     d.gated = s.gated ? 1 : 0;
     d.pos_offset = s.pos_offset;
     d.bias = s.bias;
@@ -506,8 +692,9 @@ extern "C" ra_status refadapt_gemm(const ra_gemm_args* a, void* stream) {
     }
     ra_seg as{const_cast<void*>(s.a), s.a_stride_s, 0, s.a_stride_r, s.rows, 0};
     ra_seg ws{const_cast<void*>(s.w), 0, 0, a->K, a->N, 0};
+      // The pair kernel loads 128-row boxes of A and of W (each CTA its half).
     if (!encode_seg(&p.tm_a[g], as, a->B, 1, a->K, BK, BM, true) ||
-        !encode_seg(&p.tm_w[g], ws, 1, 1, a->K, BK, BN, true))
+        !encode_seg(&p.tm_w[g], ws, 1, 1, a->K, BK, pair ? 128 : BN, true))
       return RA_EINVAL;
     tiles += int64_t(a->B) * d.m_tiles * p.n_tiles_n;
   }
@@ -517,12 +704,38 @@ extern "C" ra_status refadapt_gemm(const ra_gemm_args* a, void* stream) {
   static cudaError_t attr_err = cudaSuccess;
   std::call_once(once, [] {
     attr_err = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC);
+    if (attr_err == cudaSuccess)
+      attr_err = cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_ALLOC);
   });
   if (attr_err != cudaSuccess) {
     set_error("refadapt_gemm: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
     return RA_ECUDA;
   }
-  const int64_t grid = tiles < num_sms() ? tiles : num_sms();
-  gemm_kernel<<<unsigned(grid), THREADS, SMEM_ALLOC, static_cast<cudaStream_t>(stream)>>>(p);
+  const cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (!pair) {
+    const int64_t grid = tiles < sms ? tiles : sms;
+    gemm_kernel<<<unsigned(grid), THREADS, SMEM_ALLOC, st>>>(p);
+    return launch_status("refadapt_gemm");
+  }
+  const int64_t clusters = tiles < sms / 2 ? tiles : (sms / 2 > 0 ? sms / 2 : 1);
+  cudaLaunchConfig_t cfg;
+  std::memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3(unsigned(2 * clusters), 1, 1);
+  cfg.blockDim = dim3(THREADS, 1, 1);
+  cfg.dynamicSmemBytes = P_SMEM_ALLOC;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  const cudaError_t e = cudaLaunchKernelEx(&cfg, gemm_pair_kernel, p);
+  if (e != cudaSuccess) {
+    set_error("refadapt_gemm: pair launch failed: %s", cudaGetErrorString(e));
+    cudaGetLastError();
+    return RA_ECUDA;
+  }
   return launch_status("refadapt_gemm");
 }

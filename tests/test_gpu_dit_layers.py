@@ -75,7 +75,7 @@ def test_ln_modulate_segments_and_gating(cuda_ok, C):
             assert ok, (r, s, nbad, eq)
 
 
-def _gemm_case(B, K, N, rows_list, epi, g, gated=None, modes=None, inplace=False):
+def _gemm_case(B, K, N, rows_list, epi, g, gated=None, modes=None, inplace=False, tile_mode=0):
     from paper_2609_32415_gb300 import api
     from paper_2609_32415_gb300._lib import RA_EPI_GELU, RA_EPI_RESID, RA_EPI_STORE
     segs, keep = [], []
@@ -96,7 +96,7 @@ def _gemm_case(B, K, N, rows_list, epi, g, gated=None, modes=None, inplace=False
             keep.append((a, w, bias, None, None, sd["out"]))
         segs.append(sd)
     mode = None if modes is None else torch.tensor(modes, dtype=torch.int32, device="cuda")
-    api.refadapt_gemm(segs, N, K, epi, mode=mode)
+    api.refadapt_gemm(segs, N, K, epi, mode=mode, tile_mode=tile_mode)
     torch.cuda.synchronize()
     for i, (a, w, bias, resid, gate, out) in enumerate(keep):
         for s in range(B):
@@ -116,35 +116,44 @@ def _gemm_case(B, K, N, rows_list, epi, g, gated=None, modes=None, inplace=False
             assert ok, (epi, i, s, nbad, eq)
 
 
+# tile_mode 1: one CTA per 128 x 256 tile; 2: CTA pairs (cta_group::2) on 256 x 256 tiles.
+TILE_MODES = [1, 2]
+
+
+@pytest.mark.parametrize("tile_mode", TILE_MODES)
 @pytest.mark.parametrize("K,N,rows", [(64, 256, [1]), (256, 768, [40, 130, 77]), (3072, 512, [300]),
                                       (512, 2048, [2500])])
-def test_gemm_store_matches_oracle(cuda_ok, K, N, rows):
+def test_gemm_store_matches_oracle(cuda_ok, K, N, rows, tile_mode):
     from paper_2609_32415_gb300._lib import RA_EPI_STORE
-    _gemm_case(2, K, N, rows, RA_EPI_STORE, torch.Generator().manual_seed(K + N))
+    _gemm_case(2, K, N, rows, RA_EPI_STORE, torch.Generator().manual_seed(K + N), tile_mode=tile_mode)
 
 
-def test_gemm_gelu_matches_oracle(cuda_ok):
+@pytest.mark.parametrize("tile_mode", TILE_MODES)
+def test_gemm_gelu_matches_oracle(cuda_ok, tile_mode):
     from paper_2609_32415_gb300._lib import RA_EPI_GELU
-    _gemm_case(1, 256, 1024, [129, 200], RA_EPI_GELU, torch.Generator().manual_seed(5))
+    _gemm_case(1, 256, 1024, [129, 200], RA_EPI_GELU, torch.Generator().manual_seed(5), tile_mode=tile_mode)
 
 
+@pytest.mark.parametrize("tile_mode", TILE_MODES)
 @pytest.mark.parametrize("inplace", [False, True])
-def test_gemm_gated_residual_matches_oracle(cuda_ok, inplace):
+def test_gemm_gated_residual_matches_oracle(cuda_ok, inplace, tile_mode):
     from paper_2609_32415_gb300._lib import RA_EPI_RESID
     _gemm_case(2, 1024, 256, [40, 256, 200], RA_EPI_RESID, torch.Generator().manual_seed(6),
-               gated=[False, True, False], modes=[REUSE, COMPUTE], inplace=inplace)
+               gated=[False, True, False], modes=[REUSE, COMPUTE], inplace=inplace, tile_mode=tile_mode)
 
 
-def test_gemm_skips_gated_tiles_in_a_long_schedule(cuda_ok):
+@pytest.mark.parametrize("tile_mode", TILE_MODES)
+def test_gemm_skips_gated_tiles_in_a_long_schedule(cuda_ok, tile_mode):
     """Three segments, the middle one gated off for one sample, enough tiles
     that every CTA walks several (both accumulators, several phases)."""
     from paper_2609_32415_gb300._lib import RA_EPI_STORE
     _gemm_case(2, 192, 1024, [700, 1500, 900], RA_EPI_STORE, torch.Generator().manual_seed(7),
-               gated=[False, True, False], modes=[COMPUTE, REUSE])
+               gated=[False, True, False], modes=[COMPUTE, REUSE], tile_mode=tile_mode)
 
 
+@pytest.mark.parametrize("tile_mode", TILE_MODES)
 @pytest.mark.parametrize("H,d,modes", [(4, 64, [FULL, BOUNDARY]), (2, 128, [REUSE, COMPUTE])])
-def test_gemm_qkv_epilogue_matches_oracle(cuda_ok, H, d, modes):
+def test_gemm_qkv_epilogue_matches_oracle(cuda_ok, H, d, modes, tile_mode):
     """QKV projection with per-head RMS norm and RoPE at the rows' joint
     positions; the reference segment is gated: REUSE writes nothing,
     BOUNDARY writes only its query (K/V stay the cached ones)."""
@@ -167,7 +176,8 @@ def test_gemm_qkv_epilogue_matches_oracle(cuda_ok, H, d, modes):
         segs.append({"a": x, "w": w, "bias": bias, "q": out[0], "k": out[1], "v": out[2], "q_norm": qn,
                      "k_norm": kn, "pos_offset": pos0[r], "gated": r == "ref"})
         keep[r] = (x, w, bias, qn, kn, out)
-    api.refadapt_gemm(segs, 3 * C, C, RA_EPI_QKV, mode=mode, rope=rope, H=H, d=d, norm_eps=1e-6)
+    api.refadapt_gemm(segs, 3 * C, C, RA_EPI_QKV, mode=mode, rope=rope, H=H, d=d, norm_eps=1e-6,
+                      tile_mode=tile_mode)
     torch.cuda.synchronize()
     for r, (x, w, bias, qn, kn, out) in keep.items():
         pos = pos0[r] + np.arange(n[r])
