@@ -908,6 +908,48 @@ def cublas_context_tflops(M, K, N, reps=20):
     return 2.0 * M * N * K / ms / 1e9
 
 
+def dit_cpu_oracle_sample(wl, tables, budget_s):
+    """Time the CPU oracle's DiT block (oracle/dit.py, fp64) on a bounded
+    sample: R target rows of block 0 through the modulated LN + QKV + norm +
+    RoPE, their attention against all N keys, and the output projection + MLP.
+    Returns seconds per row for the linear part and per query row for the
+    attention, and the sample size."""
+    import numpy as np
+    import torch
+    import oracle
+    from oracle import dit as odit
+
+    def f64(t):
+        return oracle.bf16_to_f64(t.contiguous().cpu().view(torch.int16).numpy().view(np.uint16))
+
+    di, h_in, mods, weights = tables
+    W = {k: (f64(v) if k.startswith("w_") else v.double().cpu().numpy()) for k, v in weights[0]["image"].items()}
+    md = {k: v[0].double().cpu().numpy() for k, v in mods[(1, 0)]["image"].items()}
+    C = wl.H * wl.d
+    rng = np.random.default_rng(0)
+    keys = rng.standard_normal((wl.H, wl.N, wl.d)) / math.sqrt(wl.d)
+    vals = rng.standard_normal((wl.H, wl.N, wl.d)) / math.sqrt(wl.d)
+    nth = oracle.default_threads()
+    R = 4
+    while True:
+        h = f64(h_in[1]["tgt"][0, :R])
+        pos = wl.n_text + wl.n_ref + np.arange(R)
+        t0 = time.perf_counter()
+        q, _, _ = odit.qkv_project(h, md, W, pos, wl.H, wl.d)
+        t1 = time.perf_counter()
+        o, _ = oracle.joint_attention(q, keys, vals, 1.0 / math.sqrt(wl.d),
+                                      ref_range=(wl.n_text, wl.n_text + wl.n_ref), nthreads=nth)
+        t2 = time.perf_counter()
+        odit.post_attention(h, odit.round_bf16(o), md, W)
+        t3 = time.perf_counter()
+        total = t3 - t0
+        if total > budget_s / 3 or R >= 256:
+            break
+        R = min(256, max(R * 2, int(R * (budget_s / 2.5) / max(total, 1e-3))))
+    return {"lin_s_per_row": ((t1 - t0) + (t3 - t2)) / R, "attn_s_per_row": (t2 - t1) / R, "rows": R,
+            "sample_s": total, "threads": nth, "C": C}
+
+
 def main_dit(args):
     import torch
     import __graft_entry__ as ge
@@ -928,6 +970,22 @@ def main_dit(args):
     gt = main["gemm_flops"] / (main["gemm_ms"] * 1e-3) / 1e12
     at = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
     ms = main["total_ms"] / args.steps
+    cpu = None
+    if not args.no_cpu_baseline:
+        smp = dit_cpu_oracle_sample(wl, tables, args.cpu_budget_s)
+        per_step = []
+        for t in main["steps_t"]:
+            ms_t = 0.0
+            for b_modes in main["modes"][t]:
+                for m in b_modes:
+                    rows = wl.N if int(m) != 0 else wl.n_text + wl.n_tgt
+                    ms_t += 1000.0 * rows * (smp["lin_s_per_row"] + smp["attn_s_per_row"])
+            per_step.append(ms_t)
+        cpu = {"value": round(statistics.mean(per_step), 1), "unit": "ms/step", "cores": smp["threads"],
+               "kind": "oracle",
+               "sample": "fp64 DiT-block oracle, %d target rows of block 0 through LN + QKV + norm + RoPE, their "
+                         "attention against all %d keys, output projection + MLP (%.1f s); extrapolated per row to "
+                         "the executed rows of every block of the timed steps" % (smp["rows"], wl.N, smp["sample_s"])}
     line = {
         "workload": "DiT-block stack: " + WORKLOAD_NAMES[args.config] + (
             " (first %d blocks)" % wl.n_blocks if args.blocks > 0 else ""),
@@ -947,6 +1005,7 @@ def main_dit(args):
         "same_shape_cublas_tflops": round(ctx, 1),
         "peak": peaks["bf16_sustained"], "peak_kind": "%s, sustained bf16" % peaks["source"],
         "clocks": main["clocks"],
+        "cpu_baseline": cpu,
     }
     if refresh is not None:
         rms = refresh["total_ms"] / args.steps
