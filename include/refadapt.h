@@ -111,6 +111,11 @@ typedef struct {
  *                   query rows against reference keys (natural-log units).
  *  mode             device [B] int32 (ra_mode) or NULL (= every row runs).
  *  mass_partial     device [B][H][refadapt_mass_partial_len(n_text, n_tgt)].
+ *  mass_row_stride  the "sampled target-query rows" of Eq. 4 / Algorithm 1:
+ *                   0 or 1 counts every mass row; k > 1 counts rows 0, k,
+ *                   2k, ... of the target segment (and of the text segment
+ *                   when mass_rows = 1); the partials then sum the sampled
+ *                   rows only (divide by their count). O is unaffected.
  *  err_word         device int32 or NULL; bit 0 set on a device timeout.
  */
 typedef struct {
@@ -118,7 +123,7 @@ typedef struct {
   int32_t mass_rows;
   ra_seg q[3], k[3], v[3], o[3];
   float softmax_scale;
-  int32_t reserved;
+  int32_t mass_row_stride;  /* 0 or 1: every mass row; k > 1: rows 0, k, 2k, ... of each mass segment */
   const float* ref_logit_bias;
   const int32_t* mode;
   float* mass_partial;

@@ -22,9 +22,10 @@ Each function names the passage of the paper it restates:
                            Eq. 11.
 * ``attention_flops``      App. A.4 compute accounting.
 
-Readings of points the paper leaves open (all listed in the design doc):
-eps of Eq. 1 is a parameter (default 1e-6); all target rows are used (no row
-sampling); mass rows default to the target-latent rows (``mass_rows=0``), with
+Readings of points the paper leaves open:
+eps of Eq. 1 is a parameter (default 1e-6); all target rows are used unless
+``sample_stride`` k > 1 takes D and M over the rows 0, k, 2k, ...; mass rows
+default to the target-latent rows (``mass_rows=0``), with
 ``mass_rows=1`` for text + target; a score equal to theta reactivates; the
 reference query rows at a boundary block are the ones cached at the block's
 last materialisation (the stand-in for restoring the cached hidden state).
@@ -243,7 +244,7 @@ class Gate:
 
 
 def block_attention(q, k, v, mode, scale, bias=None, mass_rows=0, o_rows=None,
-                    want_o=True, nthreads=None):
+                    want_o=True, nthreads=None, sample_stride=1):
     """One block's executed joint attention for one sample (Algorithm 1 body).
 
     q, k, v: dict role -> float64 [H, n_role, d] for roles text, ref, tgt.
@@ -254,7 +255,9 @@ def block_attention(q, k, v, mode, scale, bias=None, mass_rows=0, o_rows=None,
     ``bias`` [H] is added to target-row x reference-key logits.
     ``o_rows``: optional dict role -> row indices at which to return O (all
     executed rows when None). Returns dict with O[role] (None when the role's
-    rows are not executed), row_mass[role], and M [H] (Eq. 4).
+    rows are not executed), row_mass[role], and M [H] (Eq. 4) over the mass
+    rows 0, k, 2k, ... of each counted role (k = ``sample_stride``, the
+    "sampled target-query rows"; 1 = every row).
     """
     H = q["tgt"].shape[0]
     n = {r: q[r].shape[1] if r != "ref" else k["ref"].shape[1] for r in ROLES}
@@ -288,15 +291,16 @@ def block_attention(q, k, v, mode, scale, bias=None, mass_rows=0, o_rows=None,
                                    biased[idx] if bias is not None else None, (r0, r1),
                                    want_o=want_o, nthreads=nthreads)
             out["O"][r] = o
-    out["M"] = exposure(out["row_mass"]["tgt"],
-                        out["row_mass"]["text"] if mass_rows == 1 else None)
+    kk = max(1, int(sample_stride))
+    out["M"] = exposure(out["row_mass"]["tgt"][:, ::kk],
+                        out["row_mass"]["text"][:, ::kk] if mass_rows == 1 else None)
     return out
 
 
 def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
                 scale=None, bias=None, mass_rows=0, forced_boundary=-1, tie=None,
                 o_rows=None, want_o=True, nthreads=None, cue="product", diagnostics=False,
-                diag_row_stride=1):
+                diag_row_stride=1, sample_stride=1):
     """Algorithm 1 over ``n_steps`` denoising steps and ``n_blocks`` blocks.
 
     ``get_inputs(t, b)`` returns dict role -> (q, k, v), each a uint16 array of
@@ -326,6 +330,10 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
     M_fresh (the exposure of Eq. 4 with fresh reference keys; the executed M
     is the same-step cached exposure when the block reuses).
 
+    ``sample_stride`` k > 1: D (Eq. 1) and M (Eq. 4) over the sampled target
+    query rows 0, k, 2k, ... only (Algorithm 1 stores sampled target queries
+    and masses); 1 = every row.
+
     Returns records[t][b] = dict(mode [B], gbar [B], D [B,H], M [B,H],
     O [B] of dict role -> array or None, a_b [B]) (+ the diagnostics).
     """
@@ -345,10 +353,13 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
             q_tgt = f["tgt"][0]
             H, d = q_tgt.shape[1], q_tgt.shape[3]
             sc = (1.0 / math.sqrt(d)) if scale is None else float(scale)
+            ks = max(1, int(sample_stride))
             if cue == "anchor_product":
-                D = q_change(q_tgt, anchor_q[b], eps) if (t >= 1 and anchor_q[b] is not None) else None
+                D = q_change(q_tgt[:, :, ::ks], anchor_q[b][:, :, ::ks], eps) \
+                    if (t >= 1 and anchor_q[b] is not None) else None
             else:
-                D = q_change(q_tgt, prev_q[b], eps) if (t >= 1 and prev_q[b] is not None) else None
+                D = q_change(q_tgt[:, :, ::ks], prev_q[b][:, :, ::ks], eps) \
+                    if (t >= 1 and prev_q[b] is not None) else None
             modes, gbars = gate.decide(t, b, D, prev_M[b], tie=tie)
             if anchor_q[b] is None:
                 anchor_q[b] = np.array(q_tgt)
@@ -373,7 +384,7 @@ def closed_loop(get_inputs, n_steps, n_blocks, B, *, theta, delta_max, eps=1e-6,
                 rows = o_rows(t, b, s) if o_rows is not None else None
                 res = block_attention(qd, kd, vd, mode, sc,
                                       None if bias is None else np.asarray(bias),
-                                      mass_rows, rows, want_o, nthreads)
+                                      mass_rows, rows, want_o, nthreads, sample_stride)
                 M[s] = res["M"]
                 O.append(res["O"])
                 if diagnostics:

@@ -36,7 +36,7 @@ class RaSeg(ctypes.Structure):
 class RaAttnArgs(ctypes.Structure):
     _fields_ = [("B", c_int32), ("H", c_int32), ("d", c_int32), ("mass_rows", c_int32),
                 ("q", RaSeg * 3), ("k", RaSeg * 3), ("v", RaSeg * 3), ("o", RaSeg * 3),
-                ("softmax_scale", c_float), ("reserved", c_int32),
+                ("softmax_scale", c_float), ("mass_row_stride", c_int32),
                 ("ref_logit_bias", c_void_p), ("mode", c_void_p), ("mass_partial", c_void_p),
                 ("err_word", c_void_p)]
 

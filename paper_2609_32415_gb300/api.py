@@ -51,7 +51,7 @@ def alloc_mass_partial(B, H, n_text, n_tgt, device="cuda"):
 
 
 def refadapt_joint_attn(q, k, v, o, mass_partial, mode=None, softmax_scale=0.0, ref_logit_bias=None,
-                        mass_rows=0, err_word=None, stream=None):
+                        mass_rows=0, err_word=None, mass_row_stride=0, stream=None):
     """q, k, v, o: sequences (text, ref, tgt) of [B, H, n, d] tensors; q[1] / o[1] may be None."""
     lib = _lib.load()
     B, H, _, d = k[2].shape
@@ -64,6 +64,7 @@ def refadapt_joint_attn(q, k, v, o, mass_partial, mode=None, softmax_scale=0.0, 
         a.v[r] = seg(v[r])
         a.o[r] = seg(o[r], n_q)
     a.softmax_scale = float(softmax_scale)
+    a.mass_row_stride = int(mass_row_stride)
     a.ref_logit_bias = _ptr(ref_logit_bias)
     a.mode = _ptr(mode)
     a.mass_partial = _ptr(mass_partial)

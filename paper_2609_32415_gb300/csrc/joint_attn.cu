@@ -79,6 +79,7 @@ struct Params {
   int32_t kv_tiles[3];
   int32_t B, H;
   int32_t mass_rows;
+  int32_t mass_stride;  // count mass rows 0, k, 2k, ... (k <= 1: every row)
   int32_t mpl;
   float scale_log2;
   const float* bias;
@@ -462,7 +463,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
     }
     // Per-tile mass partial: sum over the tile's mass rows of l_ref / l, in a
     // fixed order (warp butterfly, then quarters 0..3).
-    const bool in_mass = (role == 2) || (role == 0 && p.mass_rows == 1);
+    const bool in_mass = ((role == 2) || (role == 0 && p.mass_rows == 1)) &&
+                         (p.mass_stride <= 1 || grow % p.mass_stride == 0);
     float mv = (ok && valid && in_mass) ? lref * inv_l : 0.f;
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) mv += __shfl_xor_sync(0xffffffffu, mv, o);
@@ -527,6 +529,10 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
     set_error("refadapt_joint_attn: mass_rows must be 0 or 1");
     return RA_EINVAL;
   }
+  if (a->mass_row_stride < 0) {
+    set_error("refadapt_joint_attn: mass_row_stride must be >= 0");
+    return RA_EINVAL;
+  }
   if (!(a->softmax_scale >= 0.f) || std::isinf(a->softmax_scale)) {
     set_error("refadapt_joint_attn: softmax_scale must be finite and >= 0");
     return RA_EINVAL;
@@ -582,6 +588,7 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
   p.B = a->B;
   p.H = a->H;
   p.mass_rows = a->mass_rows;
+  p.mass_stride = a->mass_row_stride;
   p.mpl = refadapt_mass_partial_len(a->q[RA_TEXT].n, a->q[RA_TGT].n);
   const float scale = a->softmax_scale > 0.f ? a->softmax_scale : 1.0f / std::sqrt(float(d));
   p.scale_log2 = scale * kLog2e;

@@ -50,11 +50,16 @@ class Executor:
     (Eq. 10, refadapt_q_delta of the executed target output against it).
     Logged per step in E_K, E_V, I_KV [steps, blocks, B, H] and M_fresh_part
     [steps, blocks, B, H, tiles].
+
+    ``sample_stride`` k > 1 takes D and M over the sampled target-query rows
+    0, k, 2k, ... (Eq. 4, Algorithm 1 "sampled target queries"): D from the
+    strided target Q views, M from the attention's mass partials over those
+    rows only. k = 1 uses every row.
     """
 
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
                  mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
-                 device="cuda", cue="product", diagnostics=False, diag_row_stride=1):
+                 device="cuda", cue="product", diagnostics=False, diag_row_stride=1, sample_stride=1):
         if cue not in CUES:
             raise ValueError("unknown cue %r" % (cue,))
         self.cue = cue
@@ -72,7 +77,8 @@ class Executor:
         self.a_b = torch.full((n_blocks, B), -1, dtype=torch.int32, device=dev)
         self.mpl = api.refadapt_mass_partial_len(n_text, n_tgt)
         self.mass = torch.zeros((n_blocks, B, H, self.mpl), dtype=torch.float32, device=dev)
-        self.mass_row_count = n_tgt + (n_text if mass_rows == 1 else 0)
+        k = self.sample_stride = max(1, int(sample_stride))
+        self.mass_row_count = (n_tgt + k - 1) // k + ((n_text + k - 1) // k if mass_rows == 1 else 0)
         self.D = torch.zeros((n_blocks, B, H), dtype=torch.float32, device=dev)
         self.log_steps = int(log_steps)
         self.modes = torch.full((self.log_steps, n_blocks, B), -1, dtype=torch.int32, device=dev)
@@ -117,7 +123,9 @@ class Executor:
         have_prev = t >= 1 and self._prev_qtgt[b] is not None
         if have_prev:
             ref_q = self.anchor[b] if self.anchor is not None else self._prev_qtgt[b]
-            api.refadapt_q_delta(qt, ref_q, self.D[b], self.workspace, self.eps, stream)
+            k = self.sample_stride
+            api.refadapt_q_delta(qt[:, :, ::k, :] if k > 1 else qt, ref_q[:, :, ::k, :] if k > 1 else ref_q,
+                                 self.D[b], self.workspace, self.eps, stream)
         api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
                           q_delta=self.D[b] if have_prev else None,
                           mass_partial_prev=self.mass[b] if have_prev else None,
@@ -139,7 +147,7 @@ class Executor:
             (x["text"][2], self.cache_v[b], x["tgt"][2]),
             (out["text"], out["ref"], out["tgt"]),
             self.mass[b], mode=mode, softmax_scale=self.softmax_scale, ref_logit_bias=self.bias,
-            mass_rows=self.mass_rows, err_word=self.err, stream=stream)
+            mass_rows=self.mass_rows, err_word=self.err, mass_row_stride=self.sample_stride, stream=stream)
         if self.attn_hook is not None:
             self.attn_hook("post", t, b)
         if self.diagnostics:

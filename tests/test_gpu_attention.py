@@ -202,3 +202,32 @@ def test_attention_sampled_query_rows(cuda_ok):
             assert ok, (r, worst, nw)
         got_m = mp[s].double().sum(-1).cpu().numpy() / ns
         assert np.abs(got_m - ref["M"]).max() <= M_ABS
+
+
+@pytest.mark.parametrize("stride,mass_rows", [(3, 0), (4, 1)])
+def test_attention_sampled_mass_rows(cuda_ok, stride, mass_rows):
+    """Mass partials over the sampled target rows 0, k, 2k, ... (and text rows
+    when counted): their sum over the sampled count is the oracle's M with the
+    same sample; O is unaffected."""
+    import oracle
+    from paper_2609_32415_gb300 import api
+    n = dict(text=70, ref=300, tgt=333)
+    B, H, d = 1, 3, 128
+    segs = make_segments(B, H, d, n, gen=torch.Generator().manual_seed(31))
+    out = empty_outputs(B, H, d, n)
+    mp = torch.full((B, H, api.refadapt_mass_partial_len(n["text"], n["tgt"])), float("nan"),
+                    dtype=torch.float32, device="cuda")
+    api.refadapt_joint_attn([segs[r][0] for r in ROLES], [segs[r][1] for r in ROLES], [segs[r][2] for r in ROLES],
+                            [out[r] for r in ROLES], mp, mass_rows=mass_rows, mass_row_stride=stride)
+    torch.cuda.synchronize()
+    count = (n["tgt"] + stride - 1) // stride + ((n["text"] + stride - 1) // stride if mass_rows else 0)
+    M_gpu = mp.double().sum(-1).cpu().numpy() / count
+    from _helpers import f64
+    q = {r: f64(segs[r][0][0]) for r in ROLES}
+    k = {r: f64(segs[r][1][0]) for r in ROLES}
+    v = {r: f64(segs[r][2][0]) for r in ROLES}
+    ref = oracle.block_attention(q, k, v, FULL, 1.0 / math.sqrt(d), mass_rows=mass_rows, sample_stride=stride)
+    assert np.abs(M_gpu[0] - ref["M"]).max() < 2e-5
+    for r in ROLES:
+        ok, worst, nw = o_close(out[r][0].double().cpu().numpy(), ref["O"][r])
+        assert ok, (r, worst)

@@ -151,3 +151,47 @@ def test_closed_loop_staleness_diagnostics(cuda_ok):
                 assert ok.all(), (t, b, key, got, want)
             assert np.abs(diag["M_fresh"][t, b] - r["M_fresh"]).max() <= M_ABS, (t, b)
             assert np.abs(diag["I_KV"][t, b] - r["I_KV"]).max() <= 5e-3, (t, b, diag["I_KV"][t, b], r["I_KV"])
+
+
+def test_closed_loop_sampled_target_rows(cuda_ok):
+    """D and M over the sampled target rows 0, 4, 8, ... (Algorithm 1's
+    sampled target queries and masses) through the executor against the
+    oracle's closed loop with the same sample."""
+    from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
+    wl = synth.custom_workload(2, 4, 128, 33, 300, 200, n_blocks=4, n_steps=5, ref_drift=0.05,
+                               tgt_drift=[0.05, 0.1, 0.3, 0.4], theta=0.08, delta_max=3)
+    traj = synth.Trajectory(wl, device="cuda")
+    ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max,
+                  wl.eps, log_steps=wl.n_steps, sample_stride=4)
+    keep, D = {}, np.zeros((wl.n_steps, wl.n_blocks, wl.B, wl.H))
+    for t in range(wl.n_steps):
+        xs = []
+        for b in range(wl.n_blocks):
+            X = traj.get(t, b)
+            keep[(t, b)] = X
+            xs.append(roles_from_joint(X, wl.offsets(), wl.n))
+
+        def grab(tt, bb):
+            D[tt, bb] = ex.D[bb].double().cpu().numpy()
+
+        ex.step(t, xs, after_block=grab)
+    torch.cuda.synchronize()
+    ex.check()
+    modes = ex.modes.cpu().numpy()
+    gbar = ex.gbar.double().cpu().numpy()
+    off = wl.offsets()
+
+    def raw(t, b):
+        X = keep[(t, b)]
+        return {r: tuple(bits(X[z, :, :, off[r]:off[r] + wl.n[r], :]) for z in range(3)) for r in ROLES}
+
+    rec = oracle.closed_loop(raw, wl.n_steps, wl.n_blocks, wl.B, theta=wl.theta, delta_max=wl.delta_max,
+                             eps=wl.eps, tie=lambda t, b, s: modes[t, b, s] == 1, want_o=False, sample_stride=4)
+    for t in range(wl.n_steps):
+        for b in range(wl.n_blocks):
+            r = rec[t][b]
+            assert list(modes[t, b]) == r["mode"], (t, b, modes[t, b], r["mode"])
+            if t >= 1:
+                assert (np.abs(D[t, b] - r["D"]) / np.abs(r["D"])).max() <= D_REL, (t, b)
+                np.testing.assert_allclose(gbar[t, b], r["gbar"], rtol=1e-4, atol=1e-6)
+    assert (modes == 1).any() and (modes == 0).any()

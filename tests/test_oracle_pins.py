@@ -477,3 +477,55 @@ def test_diagnostics_match_their_definitions():
         want = np.sqrt(((a - b_) ** 2).sum(axis=(1, 2))) / (np.sqrt((b_ ** 2).sum(axis=(1, 2))) + 1e-6)
         np.testing.assert_allclose(r["I_KV"][s], want, rtol=1e-12)
         assert np.all(r["I_KV"][s] > 0)
+
+
+# --------------------------------------------------------------------------- sampled target rows
+def test_sampled_rows_mass_is_the_brute_force_mean_over_the_sample():
+    """Eq. 4 over the sampled target rows 0, k, 2k, ...: the mean of the
+    brute-force row masses of exactly those rows (text rows too when counted)."""
+    rng = np.random.default_rng(21)
+    H, d = 2, 4
+    n = {"text": 4, "ref": 5, "tgt": 7}
+    q = {r: _rand(rng, H, n[r], d) for r in oracle.ROLES}
+    k = {r: _rand(rng, H, n[r], d) for r in oracle.ROLES}
+    v = {r: _rand(rng, H, n[r], d) for r in oracle.ROLES}
+    keys = np.concatenate([k["text"], k["ref"], k["tgt"]], axis=1)
+    vals = np.concatenate([v["text"], v["ref"], v["tgt"]], axis=1)
+    r0, r1 = n["text"], n["text"] + n["ref"]
+    for mass_rows in (0, 1):
+        for ks in (1, 2, 3):
+            res = oracle.block_attention(q, k, v, FULL, 0.5, mass_rows=mass_rows, sample_stride=ks)
+            rows = []
+            for r in (("tgt", "text") if mass_rows else ("tgt",)):
+                _, m = _brute_attention(q[r].tolist(), keys.tolist(), vals.tolist(), 0.5, None, None, r0, r1)
+                rows.append(m[:, ::ks])
+            want = np.concatenate(rows, axis=1).mean(axis=1)
+            np.testing.assert_allclose(res["M"], want, rtol=1e-12)
+
+
+def test_sampled_rows_change_ignores_unsampled_rows():
+    """Eq. 1 over the sampled target rows: doubling exactly the sampled rows
+    gives D = 1/(1 + eps/||q_prev||) whatever the other rows do, while the
+    every-row D differs."""
+    rng = np.random.default_rng(22)
+    B, H, d, ks = 1, 2, 8, 3
+    n = (3, 6, 10)
+    prev = rng.standard_normal((B, H, n[2], d))
+    cur = rng.standard_normal((B, H, n[2], d))
+    cur[:, :, ::ks] = 2.0 * prev[:, :, ::ks]
+    bits = {}
+    for t, tq in ((0, prev), (1, cur)):
+        raw = {}
+        for r, nn in zip(oracle.ROLES, n):
+            z = [rng.standard_normal((B, H, nn, d)) for _ in range(3)]
+            if r == "tgt":
+                z[0] = tq
+            raw[r] = tuple(torch.from_numpy(x).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+                           for x in z)
+        bits[t] = raw
+    rec = oracle.closed_loop(lambda t, b: bits[t], 2, 1, B, theta=1e9, delta_max=10, sample_stride=ks)
+    qp = oracle.bf16_to_f64(bits[0]["tgt"][0])[:, :, ::ks]
+    want = 1.0 / (1.0 + 1e-6 / np.sqrt((qp ** 2).sum(axis=(2, 3))))
+    np.testing.assert_allclose(rec[1][0]["D"], want, rtol=1e-12)
+    full = oracle.closed_loop(lambda t, b: bits[t], 2, 1, B, theta=1e9, delta_max=10)
+    assert np.abs(full[1][0]["D"] - want).max() > 1e-2
