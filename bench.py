@@ -12,8 +12,11 @@ Timed steps cycle through the 8-step trajectory (step 0 is a full refresh),
 so --steps 8 times every step of one trajectory once. The same steps are also
 timed with an always-refresh gate (delta_max = 1) for the speedup.
 
-Prints one JSON line (rank 0). --impl reference times the CPU oracle instead
-(a bounded sample per step, extrapolated).
+Prints one JSON line (rank 0). Its "dit_stack" object times the same
+algorithm over a stack of random-weight DiT blocks around the attention (QKV,
+output projection, MLP, LayerNorms; --dit prints that measurement as its own
+line with the CPU oracle beside it; --no-dit skips it). --impl reference times
+the CPU oracle instead (a bounded sample per step, extrapolated).
 """
 import argparse
 import hashlib
@@ -62,6 +65,8 @@ def parse_args():
     ap.add_argument("--dit", action="store_true",
                     help="time the DiT-block stack (QKV / output projection / MLP GEMMs, LayerNorms and the "
                          "attention hot path) under Algorithm 1 on the workload's row partition; one JSON line")
+    ap.add_argument("--no-dit", action="store_true",
+                    help="skip the DiT-block stack summary that the default run adds to its line")
     ap.add_argument("--blocks", type=int, default=0,
                     help="run only the first N blocks of the stack (small profiling cases)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file")
@@ -592,6 +597,23 @@ def main_ours(args):
                "sample": "fp64 C oracle, %d target query rows x %d heads of block 0 (step 1) against all %d keys "
                          "(%.1f s) plus Eq. 1 over the block's target Q; extrapolated per query row to the "
                          "executed rows of the timed steps" % (s["rows"], s["heads"], wl.N, s["sample_s"])}
+    dit = None
+    if rank == 0 and ws == 1 and not args.no_dit:
+        # The DiT-block stack around the same attention (one line of its own with
+        # --dit); its inputs and weights replace the attention trajectory in HBM.
+        del inputs
+        torch.cuda.empty_cache()
+        try:
+            dit_wl = synth.make_workload(args.config)
+            if args.blocks > 0:
+                dit_wl.n_blocks = min(dit_wl.n_blocks, args.blocks)
+            d = run_dit(args, dit_wl, with_cpu=False, with_context=False)
+            dit = {k: d[k] for k in ("value", "unit", "block", "theta", "per_step_ms", "gemm_tflops",
+                                     "gemm_frac_of_bf16_peak", "gemm_share_of_step", "attn_tflops",
+                                     "always_refresh_ms_per_step", "speedup_vs_always_refresh", "clocks")
+                   if k in d}
+        except Exception as exc:  # report, do not guess
+            dit = {"error": str(exc)[:200]}
     if rank != 0:
         if ws > 1:
             dist.barrier()
@@ -659,6 +681,8 @@ def main_ours(args):
     sched = expected_schedule(wl)
     line["schedule_matches_expected"] = all(
         [int(x) for x in main["modes"][t, :, 0]] == sched[t] for t in set(main["steps_t"]))
+    if dit is not None:
+        line["dit_stack"] = dit
     emit(line, args)
     if ws > 1:
         dist.barrier()
@@ -956,14 +980,10 @@ def dit_cpu_oracle_sample(wl, tables, budget_s):
             "sample_s": total, "threads": nth, "C": C}
 
 
-def main_dit(args):
+def run_dit(args, wl, with_cpu=True, with_context=True):
+    """Time the DiT-block stack on the workload's row partition (theta
+    calibrated as below) against always-refresh; returns the summary dict."""
     import torch
-    import __graft_entry__ as ge
-    from paper_2609_32415_gb300 import synth
-    ge.build()
-    wl = synth.make_workload(args.config)
-    if args.blocks > 0:
-        wl.n_blocks = min(wl.n_blocks, args.blocks)
     peaks = load_peaks()
     tables = dit_tables(wl, "cuda")
     torch.cuda.synchronize()
@@ -972,26 +992,9 @@ def main_dit(args):
     main = time_dit(wl, tables, args.warmup, args.steps, theta, wl.delta_max, timing=True, clocks=clocks)
     refresh = None if args.no_refresh_baseline else time_dit(wl, tables, args.warmup, args.steps, theta, 1)
     C = wl.H * wl.d
-    ctx = cublas_context_tflops(wl.n_text + wl.n_ref + wl.n_tgt, C, 3 * C)
     gt = main["gemm_flops"] / (main["gemm_ms"] * 1e-3) / 1e12
     at = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
     ms = main["total_ms"] / args.steps
-    cpu = None
-    if not args.no_cpu_baseline:
-        smp = dit_cpu_oracle_sample(wl, tables, args.cpu_budget_s)
-        per_step = []
-        for t in main["steps_t"]:
-            ms_t = 0.0
-            for b_modes in main["modes"][t]:
-                for m in b_modes:
-                    rows = wl.N if int(m) != 0 else wl.n_text + wl.n_tgt
-                    ms_t += 1000.0 * rows * (smp["lin_s_per_row"] + smp["attn_s_per_row"])
-            per_step.append(ms_t)
-        cpu = {"value": round(statistics.mean(per_step), 1), "unit": "ms/step", "cores": smp["threads"],
-               "kind": "oracle",
-               "sample": "fp64 DiT-block oracle, %d target rows of block 0 through LN + QKV + norm + RoPE, their "
-                         "attention against all %d keys, output projection + MLP (%.1f s); extrapolated per row to "
-                         "the executed rows of every block of the timed steps" % (smp["rows"], wl.N, smp["sample_s"])}
     line = {
         "workload": "DiT-block stack: " + WORKLOAD_NAMES[args.config] + (
             " (first %d blocks)" % wl.n_blocks if args.blocks > 0 else ""),
@@ -1008,17 +1011,43 @@ def main_dit(args):
         "gemm_tflops": round(gt, 1), "gemm_frac_of_bf16_peak": round(gt / peaks["bf16_sustained"], 4),
         "gemm_share_of_step": round(main["gemm_ms"] / main["total_ms"], 4),
         "attn_tflops": round(at, 1), "attn_share_of_step": round(main["attn_ms"] / main["total_ms"], 4),
-        "same_shape_cublas_tflops": round(ctx, 1),
         "peak": peaks["bf16_sustained"], "peak_kind": "%s, sustained bf16" % peaks["source"],
         "clocks": main["clocks"],
-        "cpu_baseline": cpu,
     }
+    if with_context:
+        line["same_shape_cublas_tflops"] = round(cublas_context_tflops(wl.n_text + wl.n_ref + wl.n_tgt, C, 3 * C), 1)
+    if with_cpu:
+        smp = dit_cpu_oracle_sample(wl, tables, args.cpu_budget_s)
+        per_step = []
+        for t in main["steps_t"]:
+            ms_t = 0.0
+            for b_modes in main["modes"][t]:
+                for m in b_modes:
+                    rows = wl.N if int(m) != 0 else wl.n_text + wl.n_tgt
+                    ms_t += 1000.0 * rows * (smp["lin_s_per_row"] + smp["attn_s_per_row"])
+            per_step.append(ms_t)
+        line["cpu_baseline"] = {
+            "value": round(statistics.mean(per_step), 1), "unit": "ms/step", "cores": smp["threads"], "kind": "oracle",
+            "sample": "fp64 DiT-block oracle, %d target rows of block 0 through LN + QKV + norm + RoPE, their "
+                      "attention against all %d keys, output projection + MLP (%.1f s); extrapolated per row to "
+                      "the executed rows of every block of the timed steps" % (smp["rows"], wl.N, smp["sample_s"])}
     if refresh is not None:
         rms = refresh["total_ms"] / args.steps
         line["always_refresh_ms_per_step"] = round(rms, 3)
         line["speedup_vs_always_refresh"] = round(rms / ms, 3)
-    emit(line, args)
+    del tables
+    torch.cuda.empty_cache()
+    return line
 
+
+def main_dit(args):
+    import __graft_entry__ as ge
+    from paper_2609_32415_gb300 import synth
+    ge.build()
+    wl = synth.make_workload(args.config)
+    if args.blocks > 0:
+        wl.n_blocks = min(wl.n_blocks, args.blocks)
+    emit(run_dit(args, wl, with_cpu=not args.no_cpu_baseline), args)
 
 def main():
     args = parse_args()
