@@ -13,6 +13,10 @@
 //               from TMEM as the A operand of O_t += P_t V_j. Issue order per
 //               key tile: PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1), so the tensor
 //               core works on one tile while the other tile's softmax runs.
+//               Each product's K steps leave one asm block (one predicate,
+//               descriptors advanced by immediates): the issuing warp shares
+//               its SM sub-partition with two softmax warps, and the MMA rate
+//               follows the issuing thread's instruction count.
 //   warps 2..5  softmax / epilogue of tile A, warps 6..9 of tile B: thread =
 //               query row = TMEM lane (lane quarter = warp % 4). Online softmax
 //               in log2 units with a lazy rescale (the running max only moves
@@ -288,24 +292,14 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
       bool issued_any = false;
       auto qk = [&](int j, int t) {
         const int s = j % S;
-        const uint32_t d_t = tmem + C::TM_S + 128 * t;
-        const uint32_t qbase = sq + t * C::TILE_BYTES;
-#pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * C::CHUNK_BYTES + (kk & 3) * 32;
-          umma_ss(d_t, sdesc_sw128(qbase + off, 16, 1024), sdesc_sw128(sk + s * C::TILE_BYTES + off, 16, 1024),
-                  IDESC_QK, kk > 0 ? 1u : 0u);
-        }
+        umma_ss_ksteps<D / 16>(tmem + C::TM_S + 128 * t, sdesc_sw128(sq + t * C::TILE_BYTES, 16, 1024),
+                               sdesc_sw128(sk + s * C::TILE_BYTES, 16, 1024), IDESC_QK, 0u);
         umma_commit(s_full + t);
       };
       auto pv = [&](int j, int t) {
         const int s = j % S;
-        const uint32_t p_t = tmem + C::TM_S + 128 * t;
-        const uint32_t o_t = tmem + C::TM_O + 128 * t;
-#pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk)
-          umma_ts(o_t, p_t + kk * 8, sdesc_sw128(sv + s * C::TILE_BYTES + kk * 16 * 128, C::CHUNK_BYTES, 1024),
-                  IDESC_PV, (j > 0 || kk > 0) ? 1u : 0u);
+        umma_ts_ksteps8(tmem + C::TM_O + 128 * t, tmem + C::TM_S + 128 * t,
+                        sdesc_sw128(sv + s * C::TILE_BYTES, C::CHUNK_BYTES, 1024), IDESC_PV, j > 0 ? 1u : 0u);
         umma_commit(o_done + t);
       };
       bool ok = mbar_wait(q_full, 0, ctl) && mbar_wait(k_full, 0, ctl);
