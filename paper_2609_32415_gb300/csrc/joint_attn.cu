@@ -17,7 +17,10 @@
 //               descriptors advanced by immediates): the issuing warp shares
 //               its SM sub-partition with two softmax warps, and the MMA rate
 //               follows the issuing thread's instruction count.
-//   warps 2..5  softmax / epilogue of tile A, warps 6..9 of tile B: thread =
+//   warps 2, 3  idle (they complete warpgroup 0, which hands registers over:
+//               setmaxnreg 56 there, 224 in the softmax warpgroups; 4 x 56 +
+//               8 x 224 = 12 x 168, the launch allocation).
+//   warps 4..7  softmax / epilogue of tile A, warps 8..11 of tile B: thread =
 //               query row = TMEM lane (lane quarter = warp % 4). Online softmax
 //               in log2 units with a lazy rescale (the running max only moves
 //               when a tile's max exceeds it by more than 2^8), the row sum l
@@ -46,7 +49,7 @@ namespace attn {
 
 constexpr int BM = 128;  // query rows per tile (= TMEM lanes)
 constexpr int BN = 128;  // keys per tile
-constexpr int NUM_THREADS = 320;
+constexpr int NUM_THREADS = 384;
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kRescaleThresh = 8.0f;  // log2 units: p <= 2^8 between rescales
 
@@ -234,104 +237,112 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
   const uint32_t tmem = *tmem_slot;
   const WaitCtl ctl{abort_flag, p.err_word, p.budget_ns};
   const int nkv = p.kv_tiles[0] + p.kv_tiles[1] + p.kv_tiles[2];
-
-  if (warp == 0) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ TMA producer
-      tma_prefetch_desc(&p.tm_q[role]);
-      for (int r = 0; r < 3; ++r)
-        if (p.kv_tiles[r] > 0) {
-          tma_prefetch_desc(&p.tm_k[r]);
-          tma_prefetch_desc(&p.tm_v[r]);
+  // Register split: warpgroup 0 (producer, MMA issuer, two idle warps) gives
+  // up registers to the two softmax warpgroups: 4 x 56 + 8 x 224 = 12 x 168,
+  // the launch allocation.
+  if (warp < 4) {
+    setmaxnreg_dec<56>();
+    if (warp == 0) {
+      if (lane == 0) {
+        // ------------------------------------------------------------ TMA producer
+        tma_prefetch_desc(&p.tm_q[role]);
+        for (int r = 0; r < 3; ++r)
+          if (p.kv_tiles[r] > 0) {
+            tma_prefetch_desc(&p.tm_k[r]);
+            tma_prefetch_desc(&p.tm_v[r]);
+          }
+        int k_issued = 0, v_issued = 0;  // K / V tiles whose loads were issued
+        mbar_arrive_expect_tx(q_full, C::TILE_BYTES * (has_b ? 2 : 1));
+        for (int t = 0; t < (has_b ? 2 : 1); ++t)
+          for (int c = 0; c < C::CHUNKS; ++c)
+            tma_load_4d(smem + C::OFF_Q + t * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_q[role], q_full, c * 64,
+                        (tileA + t) * BM, h, b);
+        for (int j = 0; j < nkv; ++j) {
+          const int s = j % S;
+          const uint32_t ph = (j / S) & 1;
+          int r, row0;
+          kv_tile(p, j, r, row0);
+          if (j >= S && !mbar_wait(k_empty + s, ph ^ 1, ctl)) break;
+          mbar_arrive_expect_tx(k_full + s, C::TILE_BYTES);
+          for (int c = 0; c < C::CHUNKS; ++c)
+            tma_load_4d(smem + C::OFF_K + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_k[r], k_full + s,
+                        c * 64, row0, h, b);
+          ++k_issued;
+          if (j >= S && !mbar_wait(v_empty + s, ph ^ 1, ctl)) break;
+          mbar_arrive_expect_tx(v_full + s, C::TILE_BYTES);
+          for (int c = 0; c < C::CHUNKS; ++c)
+            tma_load_4d(smem + C::OFF_V + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_v[r], v_full + s,
+                        c * 64, row0, h, b);
+          ++v_issued;
         }
-      int k_issued = 0, v_issued = 0;  // K / V tiles whose loads were issued
-      mbar_arrive_expect_tx(q_full, C::TILE_BYTES * (has_b ? 2 : 1));
-      for (int t = 0; t < (has_b ? 2 : 1); ++t)
-        for (int c = 0; c < C::CHUNKS; ++c)
-          tma_load_4d(smem + C::OFF_Q + t * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_q[role], q_full, c * 64,
-                      (tileA + t) * BM, h, b);
-      for (int j = 0; j < nkv; ++j) {
-        const int s = j % S;
-        const uint32_t ph = (j / S) & 1;
-        int r, row0;
-        kv_tile(p, j, r, row0);
-        if (j >= S && !mbar_wait(k_empty + s, ph ^ 1, ctl)) break;
-        mbar_arrive_expect_tx(k_full + s, C::TILE_BYTES);
-        for (int c = 0; c < C::CHUNKS; ++c)
-          tma_load_4d(smem + C::OFF_K + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_k[r], k_full + s,
-                      c * 64, row0, h, b);
-        ++k_issued;
-        if (j >= S && !mbar_wait(v_empty + s, ph ^ 1, ctl)) break;
-        mbar_arrive_expect_tx(v_full + s, C::TILE_BYTES);
-        for (int c = 0; c < C::CHUNKS; ++c)
-          tma_load_4d(smem + C::OFF_V + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_v[r], v_full + s,
-                      c * 64, row0, h, b);
-        ++v_issued;
-      }
-      if (*abort_flag) {
-        // Let every load this thread issued land before the CTA exits: stage s
-        // received loads for j = s, s + S, ...; wait for the last one's phase.
-        mbar_wait_drain(q_full, 0, p.budget_ns);
-        for (int s = 0; s < S; ++s) {
-          const int nk = (k_issued > s) ? (k_issued - s + S - 1) / S : 0;
-          const int nv = (v_issued > s) ? (v_issued - s + S - 1) / S : 0;
-          if (nk > 0) mbar_wait_drain(k_full + s, (nk - 1) & 1, p.budget_ns);
-          if (nv > 0) mbar_wait_drain(v_full + s, (nv - 1) & 1, p.budget_ns);
+        if (*abort_flag) {
+          // Let every load this thread issued land before the CTA exits: stage s
+          // received loads for j = s, s + S, ...; wait for the last one's phase.
+          mbar_wait_drain(q_full, 0, p.budget_ns);
+          for (int s = 0; s < S; ++s) {
+            const int nk = (k_issued > s) ? (k_issued - s + S - 1) / S : 0;
+            const int nv = (v_issued > s) ? (v_issued - s + S - 1) / S : 0;
+            if (nk > 0) mbar_wait_drain(k_full + s, (nk - 1) & 1, p.budget_ns);
+            if (nv > 0) mbar_wait_drain(v_full + s, (nv - 1) & 1, p.budget_ns);
+          }
         }
       }
-    }
-  } else if (warp == 1) {
-    if (lane == 0) {
-      // ------------------------------------------------------------ MMA issuer
-      constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0, 0);  // Q, K both K-major
-      constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, D, 0, 1);   // P K-major (TMEM), V MN-major
-      const uint32_t sq = smem_u32(smem + C::OFF_Q);
-      const uint32_t sk = smem_u32(smem + C::OFF_K);
-      const uint32_t sv = smem_u32(smem + C::OFF_V);
-      const int ntile = has_b ? 2 : 1;
-      bool issued_any = false;
-      auto qk = [&](int j, int t) {
-        const int s = j % S;
-        umma_ss_ksteps<D / 16>(tmem + C::TM_S + 128 * t, sdesc_sw128(sq + t * C::TILE_BYTES, 16, 1024),
-                               sdesc_sw128(sk + s * C::TILE_BYTES, 16, 1024), IDESC_QK, 0u);
-        umma_commit(s_full + t);
-      };
-      auto pv = [&](int j, int t) {
-        const int s = j % S;
-        umma_ts_ksteps8(tmem + C::TM_O + 128 * t, tmem + C::TM_S + 128 * t,
-                        sdesc_sw128(sv + s * C::TILE_BYTES, C::CHUNK_BYTES, 1024), IDESC_PV, j > 0 ? 1u : 0u);
-        umma_commit(o_done + t);
-      };
-      bool ok = mbar_wait(q_full, 0, ctl) && mbar_wait(k_full, 0, ctl);
-      if (ok) {
-        tc_fence_after();
-        for (int t = 0; t < ntile; ++t) qk(0, t);
-        umma_commit(k_empty);
-        issued_any = true;
-      }
-      for (int j = 0; ok && j < nkv; ++j) {
-        const int s = j % S;
-        const bool next = j + 1 < nkv;
-        if (!(ok = mbar_wait(v_full + s, (j / S) & 1, ctl))) break;
-        if (next && !(ok = mbar_wait(k_full + (j + 1) % S, ((j + 1) / S) & 1, ctl))) break;
-        for (int t = 0; t < ntile; ++t) {
-          if (!(ok = mbar_wait(p_ready + t, j & 1, ctl))) break;
+    } else if (warp == 1) {
+      if (lane == 0) {
+        // ------------------------------------------------------------ MMA issuer
+        constexpr uint32_t IDESC_QK = idesc_bf16_f32(BM, BN, 0, 0);  // Q, K both K-major
+        constexpr uint32_t IDESC_PV = idesc_bf16_f32(BM, D, 0, 1);   // P K-major (TMEM), V MN-major
+        const uint32_t sq = smem_u32(smem + C::OFF_Q);
+        const uint32_t sk = smem_u32(smem + C::OFF_K);
+        const uint32_t sv = smem_u32(smem + C::OFF_V);
+        const int ntile = has_b ? 2 : 1;
+        bool issued_any = false;
+        auto qk = [&](int j, int t) {
+          const int s = j % S;
+          umma_ss_ksteps<D / 16>(tmem + C::TM_S + 128 * t, sdesc_sw128(sq + t * C::TILE_BYTES, 16, 1024),
+                                 sdesc_sw128(sk + s * C::TILE_BYTES, 16, 1024), IDESC_QK, 0u);
+          umma_commit(s_full + t);
+        };
+        auto pv = [&](int j, int t) {
+          const int s = j % S;
+          umma_ts_ksteps8(tmem + C::TM_O + 128 * t, tmem + C::TM_S + 128 * t,
+                          sdesc_sw128(sv + s * C::TILE_BYTES, C::CHUNK_BYTES, 1024), IDESC_PV, j > 0 ? 1u : 0u);
+          // O_t is read only after the last P V (the epilogue); a rescale reads it
+          // after s_full of the next tile, whose commit covers this P V too.
+          if (j + 1 == nkv) umma_commit(o_done + t);
+        };
+        bool ok = mbar_wait(q_full, 0, ctl) && mbar_wait(k_full, 0, ctl);
+        if (ok) {
           tc_fence_after();
-          pv(j, t);
-          if (next) qk(j + 1, t);  // S_t is free: PV_t(j) was issued first
+          for (int t = 0; t < ntile; ++t) qk(0, t);
+          umma_commit(k_empty);
+          issued_any = true;
         }
-        if (!ok) break;
-        umma_commit(v_empty + s);
-        if (next) umma_commit(k_empty + (j + 1) % S);
-      }
-      if (!ok && issued_any) {
-        umma_commit(drain);
-        mbar_wait_drain(drain, 0, p.budget_ns);
+        for (int j = 0; ok && j < nkv; ++j) {
+          const int s = j % S;
+          const bool next = j + 1 < nkv;
+          if (!(ok = mbar_wait(v_full + s, (j / S) & 1, ctl))) break;
+          if (next && !(ok = mbar_wait(k_full + (j + 1) % S, ((j + 1) / S) & 1, ctl))) break;
+          for (int t = 0; t < ntile; ++t) {
+            if (!(ok = mbar_wait(p_ready + t, j & 1, ctl))) break;
+            tc_fence_after();
+            pv(j, t);
+            if (next) qk(j + 1, t);  // S_t is free: PV_t(j) was issued first
+          }
+          if (!ok) break;
+          umma_commit(v_empty + s);
+          if (next) umma_commit(k_empty + (j + 1) % S);
+        }
+        if (!ok && issued_any) {
+          umma_commit(drain);
+          mbar_wait_drain(drain, 0, p.budget_ns);
+        }
       }
     }
   } else {
+    setmaxnreg_inc<224>();
     // -------------------------------------------------------------- softmax
-    const int t = (warp >= 6) ? 1 : 0;   // which Q tile this warpgroup owns
+    const int t = (warp >= 8) ? 1 : 0;   // which Q tile this warpgroup owns
     const int quarter = warp & 3;        // TMEM lane quarter this warp may access
     const int row = quarter * 32 + lane;
     const uint32_t lane_off = uint32_t(quarter * 32) << 16;
@@ -413,8 +424,8 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
       l += rs;
       if (r == 1) lref += rs;
       if (__any_sync(0xffffffffu, resc)) {
-        ok = __all_sync(0xffffffffu, mbar_wait(o_done + t, (j - 1) & 1, ctl));
-        if (!ok) break;
+        // PV_t(j-1) is complete: the commit that signalled s_full for this
+        // tile tracks every MMA issued before QK_t(j).
         tc_fence_after();
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
@@ -430,7 +441,7 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
       tc_fence_before();
       mbar_arrive(p_ready + t);
     }
-    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done + t, (nkv - 1) & 1, ctl));
+    if (ok) ok = __all_sync(0xffffffffu, mbar_wait(o_done + t, 0, ctl));
     const int grow = tile * BM + row;
     const bool valid = active && grow < p.nq[role];
     const float inv_l = 1.f / l;

@@ -215,6 +215,19 @@ __device__ __forceinline__ void umma_ts_ksteps8(uint32_t d_tmem, uint32_t a_tmem
       : "memory");
 }
 
+// Per-warp register count change (all warps of a warpgroup take the same
+// count). An increase waits until decreases elsewhere in the CTA have freed
+// enough of the launch allocation, so the counts must add up to at most the
+// launch's threads x registers.
+template <int N>
+__device__ __forceinline__ void setmaxnreg_dec() {
+  asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
+}
+template <int N>
+__device__ __forceinline__ void setmaxnreg_inc() {
+  asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;\n" ::"n"(N) : "memory");
+}
+
 // Arrive on `bar` once every tcgen05 operation this thread issued so far is done.
 __device__ __forceinline__ void umma_commit(uint64_t* bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
