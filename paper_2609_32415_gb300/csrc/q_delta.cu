@@ -262,6 +262,7 @@ struct ClusterParams {
   int64_t slab_bytes;
   int32_t bulk;
   int32_t H, rows_per_unit, per_slab, cs;
+  int32_t k_begin[CL_MAX_CS + 1];  // rank r streams units [k_begin[r], k_begin[r + 1]) of its slab
   float eps;
   float* d_out;
   uint64_t budget_ns;
@@ -269,6 +270,14 @@ struct ClusterParams {
 
 __device__ __forceinline__ void cluster_sync_all() {
   asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// Arrival that only says "this CTA has started": no release (nothing is
+// published by it; the final cluster_sync_all orders the remote stores).
+__device__ __forceinline__ void cluster_arrive() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() {
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 template <int S>
@@ -285,23 +294,28 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
   uint32_t rank;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
   const int h = blockIdx.y, b = blockIdx.z;
-  const int k0 = int(int64_t(rank) * p.per_slab / p.cs);
-  const int nu = int(int64_t(rank + 1) * p.per_slab / p.cs) - k0;
+  const int k0 = p.k_begin[rank];
+  const int nu = p.k_begin[rank + 1] - k0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  if (threadIdx.x == 0) {
-    for (int s = 0; s < CL_STAGES; ++s) {
-      mbar_init(full + s, 1);
-      mbar_init(empty + s, 1);
-    }
-    *abort_flag = 0;
-    fence_mbar_init();
-  }
-  // Every CTA of the cluster has started (its shared memory exists) before any
-  // remote store below; also orders the barrier initialisation.
-  cluster_sync_all();
+  // This CTA has started (its shared memory exists): the remote stores at the
+  // end wait for every CTA's arrival, the loads below need no one else.
+  cluster_arrive();
   const WaitCtl ctl{abort_flag, nullptr, p.budget_ns};
 
   if (warp == CL_CONSUMERS) {
+    // The producer warp sets up the ring itself and releases the consumers
+    // (named barrier 2) without waiting for them, so its first loads leave at
+    // once.
+    if (lane == 0) {
+      for (int s = 0; s < CL_STAGES; ++s) {
+        mbar_init(full + s, 1);
+        mbar_init(empty + s, 1);
+      }
+      *abort_flag = 0;
+      fence_mbar_init();
+    }
+    __syncwarp();
+    named_bar_arrive(2, L::THREADS);
     if (lane == 0) {
       // ---------------------------------------------------------- producer
       if (!p.bulk) {
@@ -337,6 +351,7 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
     }
   } else {
     // ------------------------------------------------------------ consumers
+    named_bar_sync(2, L::THREADS);  // the ring's barriers are initialised
     for (int i = warp; i < nu; i += CL_CONSUMERS) {
       const int s = i % CL_STAGES;
       if (!__all_sync(0xffffffffu, mbar_wait(full + s, (i / CL_STAGES) & 1, ctl))) break;
@@ -371,19 +386,22 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
       }
     }
     named_bar_sync(1, 32 * CL_CONSUMERS);
-    if (threadIdx.x == 0) {
-      // This CTA's share in unit order, stored into the leader's slot `rank`.
-      double td = 0.0, tp = 0.0;
-      for (int i = 0; i < nu; ++i) {
-        td += sums[2 * i];
-        tp += sums[2 * i + 1];
-      }
-      if (*abort_flag) td = NAN;
-      uint32_t remote;
-      asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(slots)), "r"(0));
-      asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank), "d"(td) : "memory");
-      asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank + 8), "d"(tp) : "memory");
+  }
+  // Every CTA of the cluster has arrived (started), so the leader's shared
+  // memory exists; then this CTA's share, in unit order, goes into the
+  // leader's slot `rank`.
+  cluster_wait();
+  if (threadIdx.x == 0) {
+    double td = 0.0, tp = 0.0;
+    for (int i = 0; i < nu; ++i) {
+      td += sums[2 * i];
+      tp += sums[2 * i + 1];
     }
+    if (*abort_flag) td = NAN;
+    uint32_t remote;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(slots)), "r"(0));
+    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank), "d"(td) : "memory");
+    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank + 8), "d"(tp) : "memory");
   }
   // All remote stores are done and visible to the leader; no CTA exits while
   // another may still write into its shared memory.
@@ -535,6 +553,7 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
       c.rows_per_unit = rows_per_unit;
       c.per_slab = per_slab;
       c.cs = best_cs;
+      for (int r = 0; r <= best_cs; ++r) c.k_begin[r] = int(int64_t(r) * per_slab / best_cs);
       c.eps = eps;
       c.d_out = d_out;
       c.budget_ns = wait_budget_ns();
