@@ -350,17 +350,27 @@ def time_graphs(wl, inputs, warmup, steps):
 
 
 def time_e2e(wl, inputs, warmup, steps):
-    """Same steps through the public API with host-resident inputs: every block's
-    Q/K/V are copied from pinned host memory on a copy stream (double-buffered,
-    overlapped with the previous block's compute), and each step's decisions
-    (modes, scores) are read back to pinned host memory."""
+    """Same steps through the public API with host-resident inputs. Per step:
+    the step's gates run first on every block's target Q (copied during the
+    previous step, behind that block's data) (Executor.gate_block: a gate
+    reads only that block's target queries, its
+    previous-step mass partials and the controller state of the blocks before
+    it); one device->host read of the step's modes (and gbar) follows, and
+    then, per block, the text Q/K/V and target K/V are copied, plus the
+    reference Q/K/V only when a sample materialises (a reusing block reads its
+    reference K/V from the cache), on a copy stream, triple-buffered and
+    overlapped with the attentions (Executor.attend_block), up to two blocks
+    ahead."""
     import torch
     from paper_2609_32415_gb300 import Executor
     T, nb = wl.n_steps, wl.n_blocks
     off = wl.offsets()
-    # Host copy of the trajectory: per (t, b) one contiguous tensor per (kind, role).
-    shapes = [((z, r), (wl.B, wl.H, wl.n[r], wl.d)) for z in range(3) for r in ROLES]
-    per_block = sum(math.prod(sh) for _, sh in shapes)
+    # Host layout per (t, b): [target Q | text Q, K, V, target K, V | reference Q, K, V]
+    parts = {"tq": [(0, "tgt")], "base": [(0, "text"), (1, "text"), (2, "text"), (1, "tgt"), (2, "tgt")],
+             "ref": [(0, "ref"), (1, "ref"), (2, "ref")]}
+    shape = {r: (wl.B, wl.H, wl.n[r], wl.d) for r in ROLES}
+    size = {k: sum(math.prod(shape[r]) for _, r in v) for k, v in parts.items()}
+    per_block = size["tq"] + size["base"] + size["ref"]
     # Page-locked host copy of the trajectory (cudaHostAlloc through torch's
     # pinned allocator), one buffer per (step, block). On the hosts used here
     # the first ~16 GB of pinned memory a process allocates copies at ~25 GB/s
@@ -369,90 +379,139 @@ def time_e2e(wl, inputs, warmup, steps):
     # it): that range is allocated first and left unused.
     parked = torch.empty(8 << 30, dtype=torch.bfloat16, pin_memory=True)
     bufs = [[torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True) for _ in range(nb)] for _ in range(T)]
+
+    def views(flat, start, kind):
+        out, o = {}, start
+        for z, r in parts[kind]:
+            out[(z, r)] = flat[o:o + math.prod(shape[r])].view(shape[r])
+            o += math.prod(shape[r])
+        return out
+
     host = []
+    o_base, o_ref = size["tq"], size["tq"] + size["base"]
     for t in range(T):
         row = []
         for b in range(nb):
             X = inputs[t][b]
-            parts, o = {}, 0
-            for key, sh in shapes:
-                z, r = key
-                h = bufs[t][b][o:o + math.prod(sh)].view(sh)
-                o += math.prod(sh)
-                h.copy_(X[z, :, :, off[r]:off[r] + wl.n[r], :])
-                parts[key] = h
-            row.append(parts)
+            v = {"tq": views(bufs[t][b], 0, "tq"), "base": views(bufs[t][b], o_base, "base"),
+                 "ref": views(bufs[t][b], o_ref, "ref")}
+            for kind in v:
+                for (z, r), h in v[kind].items():
+                    h.copy_(X[z, :, :, off[r]:off[r] + wl.n[r], :])
+            row.append({k: bufs[t][b][o:o + size[k]] for k, o in (("tq", 0), ("base", o_base), ("ref", o_ref))})
         host.append(row)
     torch.cuda.synchronize()
     dev = torch.device("cuda")
-    # Device staging: two slots with the host block layout (one copy per block),
-    # plus each block's target Q of the last two steps (read as q_{t-1}).
-    slots = [torch.empty(per_block, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-
-    def slot_views(flat):
-        views, o = {}, 0
-        for key, sh in shapes:
-            views[key] = flat[o:o + math.prod(sh)].view(sh)
-            o += math.prod(sh)
-        return views
-
-    slot_parts = [slot_views(x) for x in slots]
-    host_flat = bufs
-    keep = [[torch.empty(host[0][0][(0, "tgt")].shape, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-            for _ in range(nb)]
-    h2d = per_block * 2 * nb
+    # Device staging: each block's target Q for the current and the previous
+    # step (read as q_{t-1}), and NSLOT slots for the rest of a block.
+    tq = [[torch.empty(size["tq"], dtype=torch.bfloat16, device=dev) for _ in range(nb)] for _ in range(2)]
+    NSLOT = 3  # the copy stream may run two blocks ahead of the attentions
+    slots = [torch.empty(size["base"] + size["ref"], dtype=torch.bfloat16, device=dev) for _ in range(NSLOT)]
+    slot_v = [{**views(x, 0, "base"), **views(x, size["base"], "ref")} for x in slots]
     ex = Executor(nb, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max, wl.eps,
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T)
     comp = torch.cuda.current_stream()
     copy = torch.cuda.Stream()
-    slot_free = [torch.cuda.Event() for _ in range(2)]
-    for e in slot_free:
+    slot_free = [torch.cuda.Event() for _ in range(NSLOT)]
+    tq_free = [torch.cuda.Event() for _ in range(2)]
+    for e in slot_free + tq_free:
         e.record(comp)
     modes_host = torch.empty((nb, wl.B), dtype=torch.int32, pin_memory=True)
     gbar_host = torch.empty((nb, wl.B), dtype=torch.float32, pin_memory=True)
     d2h = modes_host.numel() * 4 + gbar_host.numel() * 4
+    decided = torch.cuda.Event()
+    h2d = [0]
+    PREFETCH = NSLOT  # blocks whose text and target K/V are copied before the step's modes are read
 
-    def one_step(t, counter):
-        for b in range(nb):
-            s = counter[0] % 2
-            counter[0] += 1
-            copy.wait_event(slot_free[s])
-            with torch.cuda.stream(copy):
-                slots[s].copy_(host_flat[t][b], non_blocking=True)
-                keep[b][t % 2].copy_(slot_parts[s][(0, "tgt")])
-                ready = torch.cuda.Event()
-                ready.record(copy)
-            comp.wait_event(ready)
-            x = {r: (keep[b][t % 2] if r == "tgt" else slot_parts[s][(0, r)], slot_parts[s][(1, r)],
-                     slot_parts[s][(2, r)]) for r in ROLES}
-            ex.block(t, b, x, ex.scratch_outputs())
-            slot_free[s].record(comp)
+    def copy_base(t, b, s):
+        copy.wait_event(slot_free[s])
+        with torch.cuda.stream(copy):
+            slots[s][:size["base"]].copy_(host[t][b]["base"], non_blocking=True)
+        h2d[0] += size["base"] * 2
+
+    tq_ready = [None, None]  # copy-stream event after a step parity's target queries (None: not copied yet)
+
+    def copy_tq(t_dst, p, b_range):
+        with torch.cuda.stream(copy):
+            for b in b_range:
+                tq[p][b].copy_(host[t_dst][b]["tq"], non_blocking=True)
+            e = torch.cuda.Event()
+            e.record(copy)
+        h2d[0] += size["tq"] * 2 * len(b_range)
+        return e
+
+    def one_step(t, counter, t_next):
         li = t % ex.log_steps
+        p = counter[1] % 2  # alternates per call (the step index may wrap)
+        counter[1] += 1
+        if tq_ready[p] is None:  # first step: nothing was prefetched
+            copy.wait_event(tq_free[p])
+            tq_ready[p] = copy_tq(t, p, range(nb))
+        comp.wait_event(tq_ready[p])
+        tq_ready[p] = None
+        for b in range(nb):
+            ex.gate_block(t, b, tq[p][b].view(shape["tgt"]), log_index=li)
+        tq_free[1 - p].record(comp)  # the gates of this step have read the previous step's queries
         modes_host.copy_(ex.modes[li], non_blocking=True)
         gbar_host.copy_(ex.gbar[li], non_blocking=True)
+        decided.record(comp)
+        first = counter[0]
+        for b in range(min(PREFETCH, nb)):
+            copy_base(t, b, (first + b) % NSLOT)
+        decided.synchronize()
+        need_ref = [bool((modes_host[b] != 0).any()) for b in range(nb)]
+        copy.wait_event(tq_free[1 - p])  # the next step's queries go where the previous step's were
+        for b in range(nb):
+            s = counter[0] % NSLOT
+            counter[0] += 1
+            if b >= PREFETCH:
+                copy_base(t, b, s)
+            with torch.cuda.stream(copy):
+                if need_ref[b]:
+                    slots[s][size["base"]:].copy_(host[t][b]["ref"], non_blocking=True)
+                    h2d[0] += size["ref"] * 2
+                ready = torch.cuda.Event()
+                ready.record(copy)
+            tq_ready[1 - p] = copy_tq(t_next, 1 - p, [b])  # the next step's target Q of this block, behind its data
+            comp.wait_event(ready)
+            sv = slot_v[s]
+            x = {"text": (sv[(0, "text")], sv[(1, "text")], sv[(2, "text")]),
+                 "ref": (sv[(0, "ref")], sv[(1, "ref")], sv[(2, "ref")]),
+                 "tgt": (tq[p][b].view(shape["tgt"]), sv[(1, "tgt")], sv[(2, "tgt")])}
+            ex.attend_block(t, b, x, ex.scratch_outputs(), log_index=li)
+            slot_free[s].record(comp)
 
-    # One untimed copy of every host block first: the first transfer from a
+    # One untimed copy of every host buffer first: the first transfer from a
     # freshly registered range also sets up its device-side translations.
     for t in range(T):
         for b in range(nb):
-            slots[0].copy_(host_flat[t][b], non_blocking=True)
+            slots[0][:per_block - size["tq"]].copy_(bufs[t][b][size["tq"]:], non_blocking=True)
+            tq[0][0].copy_(host[t][b]["tq"], non_blocking=True)
     torch.cuda.synchronize()
-    counter = [0]
+    counter = [0, 0]  # blocks, steps
+    seq = [i % T for i in range(warmup + steps + 1)]
     for i in range(warmup):
-        one_step(i % T, counter)
+        one_step(seq[i], counter, seq[i + 1])
     torch.cuda.synchronize()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record()
+    h2d[0] = 0
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
+    ev[0].record()
     for k in range(steps):
-        one_step((warmup + k) % T, counter)
-    e1.record()
+        one_step(seq[warmup + k], counter, seq[warmup + k + 1])
+        ev[k + 1].record()
     torch.cuda.synchronize()
     ex.check()
-    ms = e0.elapsed_time(e1)
-    del host, slots, keep, ex, host_flat, bufs, parked
-    return {"value": ms / steps, "unit": "ms/step", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+    ms = ev[0].elapsed_time(ev[-1])
+    per_step = [round(ev[k].elapsed_time(ev[k + 1]), 3) for k in range(steps)]
+    del host, slots, slot_v, tq, ex, bufs, parked
+    return {"value": ms / steps, "unit": "ms/step", "per_step_ms": per_step, "h2d_bytes_per_step": int(h2d[0] // steps),
+            "d2h_bytes_per_step": int(d2h),
             "host_buffers": "pinned (cudaHostAlloc), one per (step, block), allocated after a 16 GB pinned "
-                            "range left unused"}
+                            "range left unused",
+            "pipeline": "per step: the step's gates first (every block's target Q copied during the previous "
+                        "step), one read of the modes, then per block text Q/K/V + target K/V and reference "
+                        "Q/K/V only where a sample materialises, plus the next step's target Q; h2d bytes are "
+                        "the mean over the timed steps"}
 
 
 def time_q_delta(wl, inputs, reps=64):

@@ -117,9 +117,20 @@ class Executor:
     def block(self, t, b, x, out, log_index=None, stream=None):
         """Enqueue block b of step t. x: dict role -> (q, k, v) [B, H, n, d] views;
         out: dict role -> O [B, H, n, d]."""
+        self.gate_block(t, b, x["tgt"][0], log_index, stream)
+        self.attend_block(t, b, x, out, log_index, stream)
+
+    def gate_block(self, t, b, qt, log_index=None, stream=None):
+        """The decision half of block b of step t (Eq. 1 on the target query qt,
+        then Algorithm 1's gate into modes[.., b]). It reads only qt, the
+        previous step's target query and mass partials of this block and the
+        controller state left by the gates of blocks < b, so a step's gates may
+        all be enqueued before its attentions (the host can then read the
+        modes first, e.g. to skip copying reference rows a reusing block does
+        not read). The caller keeps qt alive until step t + 1's gate of this
+        block has been enqueued (it is read as q_{t-1})."""
         li = (t % self.log_steps) if log_index is None else log_index
         mode = self.modes[li, b]
-        qt = x["tgt"][0]
         have_prev = t >= 1 and self._prev_qtgt[b] is not None
         if have_prev:
             ref_q = self.anchor[b] if self.anchor is not None else self._prev_qtgt[b]
@@ -136,6 +147,16 @@ class Executor:
             # V copy is skipped: source and destination coincide).
             an = self.anchor[b]
             api.refadapt_ref_cache_update(qt, an, an, an, mode, t, None, stream=stream)
+        self._prev_qtgt[b] = qt
+
+    def attend_block(self, t, b, x, out, log_index=None, stream=None):
+        """The attention half of block b of step t, after gate_block(t, b): the
+        reference cache update (materialising samples) and the joint attention
+        with the mass partials. x[ref] is read only for samples whose mode is
+        not REUSE."""
+        li = (t % self.log_steps) if log_index is None else log_index
+        mode = self.modes[li, b]
+        qt = x["tgt"][0]
         qr, kr, vr = x["ref"]
         api.refadapt_ref_cache_update(kr, vr, self.cache_k[b], self.cache_v[b], mode, t, self.a_b[b],
                                       x_src=qr, x_cache=self.cache_x[b], stream=stream)
@@ -152,7 +173,6 @@ class Executor:
             self.attn_hook("post", t, b)
         if self.diagnostics:
             self._diagnose(t, b, li, x, out, stream)
-        self._prev_qtgt[b] = qt
 
     def _diagnose(self, t, b, li, x, out, stream):
         k = self.diag_row_stride
