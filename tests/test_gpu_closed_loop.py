@@ -195,3 +195,63 @@ def test_closed_loop_sampled_target_rows(cuda_ok):
                 assert (np.abs(D[t, b] - r["D"]) / np.abs(r["D"])).max() <= D_REL, (t, b)
                 np.testing.assert_allclose(gbar[t, b], r["gbar"], rtol=1e-4, atol=1e-6)
     assert (modes == 1).any() and (modes == 0).any()
+
+
+def test_gates_first_matches_block_order(cuda_ok):
+    """A step's gates enqueued before its attentions (Executor.gate_block for
+    every block, then Executor.attend_block; the order bench.py's end-to-end
+    timing uses to read the modes before copying reference rows) give the
+    same modes, gbar, M, D, mass partials and outputs, bit for bit, as the
+    block-by-block order: a gate reads nothing an attention of the same step
+    writes. Reusing blocks get garbage reference rows here, which they must
+    not read."""
+    from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
+    wl = synth.custom_workload(2, 4, 128, 33, 300, 200, n_blocks=5, n_steps=6, ref_drift=0.05,
+                               tgt_drift=[0.05, 0.1, 0.2, 0.3, 0.4], theta=0.08, delta_max=3)
+    traj = synth.Trajectory(wl, device="cuda")
+
+    def run(gates_first):
+        ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max,
+                      wl.eps, mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
+                      log_steps=wl.n_steps)
+        outs, mass, D = [], [], []
+        for t in range(wl.n_steps):
+            xs = [roles_from_joint(traj.get(t, b), wl.offsets(), wl.n) for b in range(wl.n_blocks)]
+            os_ = [{r: torch.full((wl.B, wl.H, wl.n[r], wl.d), float("nan"), dtype=torch.bfloat16, device="cuda")
+                    for r in ROLES} for _ in range(wl.n_blocks)]
+            if gates_first:
+                for b in range(wl.n_blocks):
+                    ex.gate_block(t, b, xs[b]["tgt"][0])
+                torch.cuda.synchronize()
+                modes = ex.modes[t].cpu()
+                for b in range(wl.n_blocks):
+                    x = dict(xs[b])
+                    if not bool((modes[b] != 0).any()):
+                        x["ref"] = tuple(torch.randn_like(z, dtype=torch.float32).to(torch.bfloat16)
+                                         for z in xs[b]["ref"])
+                    ex.attend_block(t, b, x, os_[b])
+                    D.append(ex.D[b].clone())
+                    mass.append(ex.mass[b].clone())
+            else:
+                for b in range(wl.n_blocks):
+                    ex.block(t, b, xs[b], os_[b])
+                    D.append(ex.D[b].clone())
+                    mass.append(ex.mass[b].clone())
+            outs.append(os_)
+        torch.cuda.synchronize()
+        ex.check()
+        return ex.modes.clone(), ex.gbar.clone(), ex.M.clone(), D, mass, outs
+
+    def same(x, y):  # bit-equal, NaN where the other has NaN (gbar has none on a step without a score)
+        return torch.equal(torch.isnan(x), torch.isnan(y)) and torch.equal(torch.nan_to_num(x), torch.nan_to_num(y))
+
+    a, b_ = run(False), run(True)
+    for x, y in zip(a[:3], b_[:3]):
+        assert same(x, y)
+    for x, y in zip(a[3] + a[4], b_[3] + b_[4]):
+        assert same(x, y)
+    for oa, ob in zip(a[5], b_[5]):
+        for ba, bb in zip(oa, ob):
+            for r in ROLES:
+                assert torch.equal(torch.nan_to_num(ba[r], 7.0), torch.nan_to_num(bb[r], 7.0)), r
+    assert (a[0] == 0).any() and (a[0] == 3).any()
