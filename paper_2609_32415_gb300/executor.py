@@ -59,7 +59,8 @@ class Executor:
 
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
                  mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
-                 device="cuda", cue="product", diagnostics=False, diag_row_stride=1, sample_stride=1):
+                 device="cuda", cue="product", diagnostics=False, diag_row_stride=1, sample_stride=1,
+                 overlap=True):
         if cue not in CUES:
             raise ValueError("unknown cue %r" % (cue,))
         self.cue = cue
@@ -86,6 +87,22 @@ class Executor:
         self.M = torch.zeros((self.log_steps, n_blocks, B, H), dtype=torch.float32, device=dev)
         self.workspace = api.q_delta_workspace(B, H, dev)
         self.state = api.new_state(B, dev)
+        # overlap: step() runs each block's decision (Q change, gate) and cache
+        # update on a side stream one block ahead, in the previous attention's
+        # tail wave (SMs its last wave leaves idle); see step().
+        self.overlap = bool(overlap)
+        if self.overlap:
+            # The attentions run on a high-priority stream and the side work on
+            # a default-priority one: the CTA scheduler serves pending attention
+            # CTAs first, so the side kernels take only SMs the attention leaves
+            # idle.
+            lo, hi = torch.cuda.Stream.priority_range()
+            self._main = torch.cuda.Stream(device=dev, priority=hi)
+            self._side = torch.cuda.Stream(device=dev, priority=lo)
+            self._fork = torch.cuda.Event()
+            self._join = torch.cuda.Event()
+            self._decided = [torch.cuda.Event() for _ in range(n_blocks)]
+            self._attn_done = [torch.cuda.Event() for _ in range(n_blocks)]
         self.err = torch.zeros(1, dtype=torch.int32, device=dev)
         self._prev_qtgt = [None] * n_blocks
         self.anchor = (torch.zeros((n_blocks, B, H, n_tgt, d), dtype=torch.bfloat16, device=dev)
@@ -93,6 +110,7 @@ class Executor:
         self.diagnostics = bool(diagnostics)
         self.diag_row_stride = int(diag_row_stride)
         if self.diagnostics:
+            self.workspace_diag = api.q_delta_workspace(B, H, dev)  # diagnostics run beside the side stream
             k = self.diag_row_stride
             n_s = (n_tgt + k - 1) // k
             self.n_tgt_sampled = n_s
@@ -154,12 +172,24 @@ class Executor:
         reference cache update (materialising samples) and the joint attention
         with the mass partials. x[ref] is read only for samples whose mode is
         not REUSE."""
+        self.update_cache(t, b, x, log_index, stream)
+        self.attend(t, b, x, out, log_index, stream)
+
+    def update_cache(self, t, b, x, log_index=None, stream=None):
+        """Block b's reference cache update of step t (after its gate):
+        materialising samples copy their reference K, V and query into the
+        cache slot and stamp a_b = t."""
+        li = (t % self.log_steps) if log_index is None else log_index
+        qr, kr, vr = x["ref"]
+        api.refadapt_ref_cache_update(kr, vr, self.cache_k[b], self.cache_v[b], self.modes[li, b], t, self.a_b[b],
+                                      x_src=qr, x_cache=self.cache_x[b], stream=stream)
+
+    def attend(self, t, b, x, out, log_index=None, stream=None):
+        """Block b's joint attention of step t (after its gate and cache
+        update), with the mass partials the next step's gate reads."""
         li = (t % self.log_steps) if log_index is None else log_index
         mode = self.modes[li, b]
         qt = x["tgt"][0]
-        qr, kr, vr = x["ref"]
-        api.refadapt_ref_cache_update(kr, vr, self.cache_k[b], self.cache_v[b], mode, t, self.a_b[b],
-                                      x_src=qr, x_cache=self.cache_x[b], stream=stream)
         if self.attn_hook is not None:
             self.attn_hook("pre", t, b)
         api.refadapt_joint_attn(
@@ -177,25 +207,61 @@ class Executor:
     def _diagnose(self, t, b, li, x, out, stream):
         k = self.diag_row_stride
         qr, kr, vr = x["ref"]
-        api.refadapt_q_delta(kr, self.cache_k[b], self.E_K[li, b], self.workspace, self.eps, stream)
-        api.refadapt_q_delta(vr, self.cache_v[b], self.E_V[li, b], self.workspace, self.eps, stream)
+        api.refadapt_q_delta(kr, self.cache_k[b], self.E_K[li, b], self.workspace_diag, self.eps, stream)
+        api.refadapt_q_delta(vr, self.cache_v[b], self.E_V[li, b], self.workspace_diag, self.eps, stream)
         q_s = x["tgt"][0][:, :, ::k, :]
         api.refadapt_joint_attn(
             (x["text"][0], None, q_s), (x["text"][1], kr, x["tgt"][1]), (x["text"][2], vr, x["tgt"][2]),
             (self._o_fresh["text"], None, self._o_fresh["tgt"]), self.M_fresh_part[li, b],
             softmax_scale=self.softmax_scale, ref_logit_bias=self.bias, err_word=self.err, stream=stream)
-        api.refadapt_q_delta(out["tgt"][:, :, ::k, :], self._o_fresh["tgt"], self.I_KV[li, b], self.workspace,
+        api.refadapt_q_delta(out["tgt"][:, :, ::k, :], self._o_fresh["tgt"], self.I_KV[li, b], self.workspace_diag,
                              self.eps, stream)
 
     def step(self, t, inputs, outs=None, log_index=None, stream=None, after_block=None):
         """Enqueue one denoising step. inputs[b]: dict role -> (q, k, v);
         outs[b] (optional): dict role -> O. The caller keeps step t's target Q
-        alive until step t + 1 has been enqueued (it is read as q_{t-1})."""
+        alive until step t + 1 has been enqueued (it is read as q_{t-1}).
+
+        With overlap (the default) block b's decision (Q change, gate) and
+        cache update run on a side stream, ordered after the step's start and
+        after the attention of block b - 2, and block b's attention waits for
+        them: so they run during the attention of block b - 1, whose last wave
+        leaves SMs idle (the attentions run on a higher-priority stream, so
+        their pending CTAs go first). Both streams fork from the caller's
+        stream at the step's start and join it at the end. A gate reads only its block's target queries, the
+        block's previous-step mass partials and the controller state of the
+        blocks before it, never an attention of the same step, so the results
+        are those of the one-stream order. Every event is recorded inside the
+        step, which can be captured as a CUDA graph."""
+        if not self.overlap:
+            for b in range(self.n_blocks):
+                out = outs[b] if outs is not None else self.scratch_outputs()
+                self.block(t, b, inputs[b], out, log_index, stream)
+                if after_block is not None:
+                    after_block(t, b)
+            return
+        caller = torch.cuda.current_stream() if stream is None else stream
+        main, side = self._main, self._side
+        self._fork.record(caller)
+        main.wait_event(self._fork)
+        side.wait_event(self._fork)  # everything enqueued before this step (the previous step's attentions)
         for b in range(self.n_blocks):
             out = outs[b] if outs is not None else self.scratch_outputs()
-            self.block(t, b, inputs[b], out, log_index, stream)
+            if b >= 2:
+                side.wait_event(self._attn_done[b - 2])
+            with torch.cuda.stream(side):
+                self.gate_block(t, b, inputs[b]["tgt"][0], log_index)
+                self.update_cache(t, b, inputs[b], log_index)
+                self._decided[b].record(side)
+            with torch.cuda.stream(main):
+                main.wait_event(self._decided[b])
+                self.attend(t, b, inputs[b], out, log_index)
+                self._attn_done[b].record(main)
             if after_block is not None:
-                after_block(t, b)
+                with torch.cuda.stream(main):
+                    after_block(t, b)
+        self._join.record(main)  # the side stream's last work is behind main's last wait
+        caller.wait_event(self._join)
 
     def capture_step(self, t, inputs, outs=None, log_index=None):
         """Capture step t (every block's launches, on one stream) as a CUDA graph.
