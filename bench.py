@@ -310,11 +310,28 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
            "gbar": ex.gbar.cpu().numpy(), "launches": launches, "clocks": clk,
            "steps_t": [(warmup + k) % T for k in range(steps)]}
     if attn_timing:
-        flops, ms = 0, 0.0
+        # Consecutive attentions may overlap (two streams): the attention time
+        # is the union of the launches' [start, end] intervals, every event
+        # read against the step's first event (the time at least one attention
+        # kernel runs); the plain sum of launch durations is kept beside it.
+        flops, ms_sum, iv = 0, 0.0, []
         for (t, b, (e0, e1)) in ev:
-            ms += e0.elapsed_time(e1)
+            ms_sum += e0.elapsed_time(e1)
+            iv.append((step_ev[0].elapsed_time(e0), step_ev[0].elapsed_time(e1)))
             flops += sum(attn_flops(wl, m) for m in modes[t, b])
-        res["attn_ms"] = ms
+        iv.sort()
+        busy, cur_a, cur_b = 0.0, None, None
+        for a, b_ in iv:
+            if cur_b is None or a > cur_b:
+                if cur_b is not None:
+                    busy += cur_b - cur_a
+                cur_a, cur_b = a, b_
+            else:
+                cur_b = max(cur_b, b_)
+        if cur_b is not None:
+            busy += cur_b - cur_a
+        res["attn_ms"] = busy
+        res["attn_ms_sum_of_launches"] = ms_sum
         res["attn_flops"] = flops
         res["attn_launches"] = len(ev)
     del ex

@@ -301,6 +301,11 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
   // end wait for every CTA's arrival, the loads below need no one else.
   cluster_arrive();
   const WaitCtl ctl{abort_flag, nullptr, p.budget_ns};
+  // Programmatic dependent launch: this grid may start while the previous
+  // kernel of the stream finishes. Each role waits for that kernel (complete,
+  // its writes visible) before it touches global memory; the next kernel of
+  // the stream may start its own set-up as soon as every CTA got here.
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
   if (warp == CL_CONSUMERS) {
     // The producer warp sets up the ring itself and releases the consumers
@@ -316,6 +321,7 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
     }
     __syncwarp();
     named_bar_arrive(2, L::THREADS);
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     if (lane == 0) {
       // ---------------------------------------------------------- producer
       if (!p.bulk) {
@@ -352,6 +358,7 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
   } else {
     // ------------------------------------------------------------ consumers
     named_bar_sync(2, L::THREADS);  // the ring's barriers are initialised
+    asm volatile("griddepcontrol.wait;" ::: "memory");  // orders the final store of D
     for (int i = warp; i < nu; i += CL_CONSUMERS) {
       const int s = i % CL_STAGES;
       if (!__all_sync(0xffffffffu, mbar_wait(full + s, (i / CL_STAGES) & 1, ctl))) break;
@@ -566,13 +573,17 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
       cfg.blockDim = dim3(best_s == 8 ? qd::ClLayout<8>::THREADS : qd::ClLayout<4>::THREADS, 1, 1);
       cfg.dynamicSmemBytes = best_s == 8 ? qd::ClLayout<8>::ALLOC : qd::ClLayout<4>::ALLOC;
       cfg.stream = static_cast<cudaStream_t>(stream);
-      cudaLaunchAttribute attr[1];
+      cudaLaunchAttribute attr[2];
       attr[0].id = cudaLaunchAttributeClusterDimension;
       attr[0].val.clusterDim.x = best_cs;
       attr[0].val.clusterDim.y = 1;
       attr[0].val.clusterDim.z = 1;
+      // may overlap the previous kernel's tail (the kernel waits for it with
+      // griddepcontrol.wait before touching global memory)
+      attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+      attr[1].val.programmaticStreamSerializationAllowed = 1;
       cfg.attrs = attr;
-      cfg.numAttrs = 1;
+      cfg.numAttrs = 2;
       const cudaError_t e = best_s == 8 ? cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel<8>, c)
                                         : cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel<4>, c);
       if (e != cudaSuccess) {

@@ -96,11 +96,14 @@ class Executor:
             # a default-priority one: the CTA scheduler serves pending attention
             # CTAs first, so the side kernels take only SMs the attention leaves
             # idle.
+            # Consecutive blocks' attentions alternate between two such
+            # streams: they share no data, so block b + 1's first CTAs may take
+            # the SMs block b's last wave leaves idle.
             lo, hi = torch.cuda.Stream.priority_range()
-            self._main = torch.cuda.Stream(device=dev, priority=hi)
+            self._mains = [torch.cuda.Stream(device=dev, priority=hi) for _ in range(2)]
             self._side = torch.cuda.Stream(device=dev, priority=lo)
             self._fork = torch.cuda.Event()
-            self._join = torch.cuda.Event()
+            self._join = [torch.cuda.Event() for _ in range(2)]
             self._decided = [torch.cuda.Event() for _ in range(n_blocks)]
             self._attn_done = [torch.cuda.Event() for _ in range(n_blocks)]
         self.err = torch.zeros(1, dtype=torch.int32, device=dev)
@@ -110,7 +113,8 @@ class Executor:
         self.diagnostics = bool(diagnostics)
         self.diag_row_stride = int(diag_row_stride)
         if self.diagnostics:
-            self.workspace_diag = api.q_delta_workspace(B, H, dev)  # diagnostics run beside the side stream
+            # diagnostics run on the attention streams: one set per block parity
+            self.workspace_diag = [api.q_delta_workspace(B, H, dev) for _ in range(2)]
             k = self.diag_row_stride
             n_s = (n_tgt + k - 1) // k
             self.n_tgt_sampled = n_s
@@ -120,17 +124,19 @@ class Executor:
             self.mpl_fresh = api.refadapt_mass_partial_len(n_text, n_s)
             self.M_fresh_part = torch.zeros((self.log_steps, n_blocks, B, H, self.mpl_fresh), dtype=torch.float32,
                                             device=dev)
-            self._o_fresh = {"text": torch.empty((B, H, n_text, d), dtype=torch.bfloat16, device=dev),
-                             "tgt": torch.empty((B, H, n_s, d), dtype=torch.bfloat16, device=dev)}
-        self._out = None
+            self._o_fresh = [{"text": torch.empty((B, H, n_text, d), dtype=torch.bfloat16, device=dev),
+                              "tgt": torch.empty((B, H, n_s, d), dtype=torch.bfloat16, device=dev)} for _ in range(2)]
+        self._out = [None, None]
         self.attn_hook = None   # optional callable(phase in {"pre", "post"}, t, b), e.g. CUDA events
 
-    def scratch_outputs(self):
-        """One shared set of O buffers (text, ref, tgt) reused by every block."""
-        if self._out is None:
-            self._out = {r: torch.empty((self.B, self.H, self.n[r], self.d), dtype=torch.bfloat16,
-                                        device=self.cache_k.device) for r in ROLES}
-        return self._out
+    def scratch_outputs(self, parity=0):
+        """A set of O buffers (text, ref, tgt) reused by every block of one
+        parity (step() gives blocks of the two parities different sets: their
+        attentions may run at the same time)."""
+        if self._out[parity] is None:
+            self._out[parity] = {r: torch.empty((self.B, self.H, self.n[r], self.d), dtype=torch.bfloat16,
+                                                device=self.cache_k.device) for r in ROLES}
+        return self._out[parity]
 
     def block(self, t, b, x, out, log_index=None, stream=None):
         """Enqueue block b of step t. x: dict role -> (q, k, v) [B, H, n, d] views;
@@ -206,16 +212,16 @@ class Executor:
 
     def _diagnose(self, t, b, li, x, out, stream):
         k = self.diag_row_stride
+        ws, of = self.workspace_diag[b % 2], self._o_fresh[b % 2]
         qr, kr, vr = x["ref"]
-        api.refadapt_q_delta(kr, self.cache_k[b], self.E_K[li, b], self.workspace_diag, self.eps, stream)
-        api.refadapt_q_delta(vr, self.cache_v[b], self.E_V[li, b], self.workspace_diag, self.eps, stream)
+        api.refadapt_q_delta(kr, self.cache_k[b], self.E_K[li, b], ws, self.eps, stream)
+        api.refadapt_q_delta(vr, self.cache_v[b], self.E_V[li, b], ws, self.eps, stream)
         q_s = x["tgt"][0][:, :, ::k, :]
         api.refadapt_joint_attn(
             (x["text"][0], None, q_s), (x["text"][1], kr, x["tgt"][1]), (x["text"][2], vr, x["tgt"][2]),
-            (self._o_fresh["text"], None, self._o_fresh["tgt"]), self.M_fresh_part[li, b],
+            (of["text"], None, of["tgt"]), self.M_fresh_part[li, b],
             softmax_scale=self.softmax_scale, ref_logit_bias=self.bias, err_word=self.err, stream=stream)
-        api.refadapt_q_delta(out["tgt"][:, :, ::k, :], self._o_fresh["tgt"], self.I_KV[li, b], self.workspace_diag,
-                             self.eps, stream)
+        api.refadapt_q_delta(out["tgt"][:, :, ::k, :], of["tgt"], self.I_KV[li, b], ws, self.eps, stream)
 
     def step(self, t, inputs, outs=None, log_index=None, stream=None, after_block=None):
         """Enqueue one denoising step. inputs[b]: dict role -> (q, k, v);
@@ -226,27 +232,32 @@ class Executor:
         cache update run on a side stream, ordered after the step's start and
         after the attention of block b - 2, and block b's attention waits for
         them: so they run during the attention of block b - 1, whose last wave
-        leaves SMs idle (the attentions run on a higher-priority stream, so
-        their pending CTAs go first). Both streams fork from the caller's
-        stream at the step's start and join it at the end. A gate reads only its block's target queries, the
+        leaves SMs idle (the attentions run on higher-priority streams, so
+        their pending CTAs go first). Consecutive attentions alternate between
+        two streams: they share no data (inputs, cache slot, outputs and mass
+        partials are the block's own), so block b + 1's first CTAs may start in
+        block b's last wave. Every stream forks from the caller's stream at
+        the step's start and joins it at the end. A gate reads only its block's target queries, the
         block's previous-step mass partials and the controller state of the
         blocks before it, never an attention of the same step, so the results
         are those of the one-stream order. Every event is recorded inside the
         step, which can be captured as a CUDA graph."""
         if not self.overlap:
             for b in range(self.n_blocks):
-                out = outs[b] if outs is not None else self.scratch_outputs()
+                out = outs[b] if outs is not None else self.scratch_outputs(b % 2)
                 self.block(t, b, inputs[b], out, log_index, stream)
                 if after_block is not None:
                     after_block(t, b)
             return
         caller = torch.cuda.current_stream() if stream is None else stream
-        main, side = self._main, self._side
+        side = self._side
         self._fork.record(caller)
-        main.wait_event(self._fork)
+        for m in self._mains:
+            m.wait_event(self._fork)
         side.wait_event(self._fork)  # everything enqueued before this step (the previous step's attentions)
         for b in range(self.n_blocks):
-            out = outs[b] if outs is not None else self.scratch_outputs()
+            main = self._mains[b % 2]
+            out = outs[b] if outs is not None else self.scratch_outputs(b % 2)
             if b >= 2:
                 side.wait_event(self._attn_done[b - 2])
             with torch.cuda.stream(side):
@@ -260,8 +271,9 @@ class Executor:
             if after_block is not None:
                 with torch.cuda.stream(main):
                     after_block(t, b)
-        self._join.record(main)  # the side stream's last work is behind main's last wait
-        caller.wait_event(self._join)
+        for m, j in zip(self._mains, self._join):  # the side stream's last work is behind a main wait
+            j.record(m)
+            caller.wait_event(j)
 
     def capture_step(self, t, inputs, outs=None, log_index=None):
         """Capture step t (every block's launches, on one stream) as a CUDA graph.
