@@ -377,7 +377,8 @@ def time_e2e(wl, inputs, warmup, steps):
     reference Q/K/V only when a sample materialises (a reusing block reads its
     reference K/V from the cache), on a copy stream, triple-buffered and
     overlapped with the attentions (Executor.attend_block), up to two blocks
-    ahead."""
+    ahead; consecutive attentions alternate between two high-priority
+    streams."""
     import torch
     from paper_2609_32415_gb300 import Executor
     T, nb = wl.n_steps, wl.n_blocks
@@ -429,6 +430,12 @@ def time_e2e(wl, inputs, warmup, steps):
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T)
     comp = torch.cuda.current_stream()
     copy = torch.cuda.Stream()
+    # consecutive blocks' attentions on two high-priority streams (as in
+    # Executor.step): block b + 1 may start in block b's last wave
+    lo_pri, hi_pri = torch.cuda.Stream.priority_range()
+    attn_streams = [torch.cuda.Stream(priority=hi_pri) for _ in range(2)]
+    gates_done = torch.cuda.Event()
+    attn_join = [torch.cuda.Event() for _ in range(2)]
     slot_free = [torch.cuda.Event() for _ in range(NSLOT)]
     tq_free = [torch.cuda.Event() for _ in range(2)]
     for e in slot_free + tq_free:
@@ -475,6 +482,9 @@ def time_e2e(wl, inputs, warmup, steps):
         first = counter[0]
         for b in range(min(PREFETCH, nb)):
             copy_base(t, b, (first + b) % NSLOT)
+        gates_done.record(comp)
+        for st in attn_streams:
+            st.wait_event(gates_done)
         decided.synchronize()
         need_ref = [bool((modes_host[b] != 0).any()) for b in range(nb)]
         copy.wait_event(tq_free[1 - p])  # the next step's queries go where the previous step's were
@@ -490,13 +500,18 @@ def time_e2e(wl, inputs, warmup, steps):
                 ready = torch.cuda.Event()
                 ready.record(copy)
             tq_ready[1 - p] = copy_tq(t_next, 1 - p, [b])  # the next step's target Q of this block, behind its data
-            comp.wait_event(ready)
+            st = attn_streams[b % 2]
+            st.wait_event(ready)
             sv = slot_v[s]
             x = {"text": (sv[(0, "text")], sv[(1, "text")], sv[(2, "text")]),
                  "ref": (sv[(0, "ref")], sv[(1, "ref")], sv[(2, "ref")]),
                  "tgt": (tq[p][b].view(shape["tgt"]), sv[(1, "tgt")], sv[(2, "tgt")])}
-            ex.attend_block(t, b, x, ex.scratch_outputs(), log_index=li)
-            slot_free[s].record(comp)
+            with torch.cuda.stream(st):
+                ex.attend_block(t, b, x, ex.scratch_outputs(b % 2), log_index=li)
+                slot_free[s].record(st)
+        for st, j in zip(attn_streams, attn_join):  # the next step's gates read this step's mass partials
+            j.record(st)
+            comp.wait_event(j)
 
     # One untimed copy of every host buffer first: the first transfer from a
     # freshly registered range also sets up its device-side translations.
