@@ -255,3 +255,49 @@ def test_gates_first_matches_block_order(cuda_ok):
             for r in ROLES:
                 assert torch.equal(torch.nan_to_num(ba[r], 7.0), torch.nan_to_num(bb[r], 7.0)), r
     assert (a[0] == 0).any() and (a[0] == 3).any()
+
+
+def test_two_stream_step_matches_one_stream(cuda_ok):
+    """Executor.step with overlap (each block's gate and cache update on a
+    side stream, consecutive attentions on two streams) gives the same modes,
+    gbar, M, D, mass partials and outputs, bit for bit, as the one-stream
+    order: no launch of the overlapped schedule reads or writes anything early
+    or late."""
+    from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
+    wl = synth.custom_workload(2, 4, 128, 33, 300, 200, n_blocks=5, n_steps=6, ref_drift=0.05,
+                               tgt_drift=[0.05, 0.1, 0.2, 0.3, 0.4], theta=0.08, delta_max=3)
+    traj = synth.Trajectory(wl, device="cuda")
+
+    def run(overlap):
+        ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max,
+                      wl.eps, mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
+                      log_steps=wl.n_steps, overlap=overlap)
+        outs, mass, D = [], [], []
+        for t in range(wl.n_steps):
+            xs = [roles_from_joint(traj.get(t, b), wl.offsets(), wl.n) for b in range(wl.n_blocks)]
+            os_ = [{r: torch.full((wl.B, wl.H, wl.n[r], wl.d), float("nan"), dtype=torch.bfloat16, device="cuda")
+                    for r in ROLES} for _ in range(wl.n_blocks)]
+
+            def grab(tt, bb):
+                D.append(ex.D[bb].clone())
+                mass.append(ex.mass[bb].clone())
+
+            ex.step(t, xs, os_, after_block=grab)
+            outs.append(os_)
+        torch.cuda.synchronize()
+        ex.check()
+        return ex.modes.clone(), ex.gbar.clone(), ex.M.clone(), D, mass, outs
+
+    def same(x, y):
+        return torch.equal(torch.isnan(x), torch.isnan(y)) and torch.equal(torch.nan_to_num(x), torch.nan_to_num(y))
+
+    a, b_ = run(False), run(True)
+    for x, y in zip(a[:3], b_[:3]):
+        assert same(x, y)
+    for x, y in zip(a[3] + a[4], b_[3] + b_[4]):
+        assert same(x, y)
+    for oa, ob in zip(a[5], b_[5]):
+        for ba, bb in zip(oa, ob):
+            for r in ROLES:
+                assert same(ba[r].float(), bb[r].float()), r
+    assert (a[0] == 0).any() and (a[0] == 3).any()
