@@ -1,6 +1,9 @@
 """Algorithm 1's host loop over the C ABI: one denoising step = for each block,
-Q change -> gate -> cache materialisation -> joint attention, all enqueued on
-one stream with the decisions kept on the device (no host sync inside a step).
+Q change -> gate -> cache materialisation -> joint attention, enqueued with the
+decisions kept on the device (no host sync inside a step). By default a block's
+decision and cache update run on a side stream beside the previous block's
+attention, and consecutive attentions alternate between two streams (see
+Executor.step); overlap=False keeps every launch on the caller's stream.
 
 Per block b the executor owns the cache state of paper Eq. 11: reference K and
 V, the cached reference hidden state (here the reference query, which is what
@@ -55,6 +58,11 @@ class Executor:
     0, k, 2k, ... (Eq. 4, Algorithm 1 "sampled target queries"): D from the
     strided target Q views, M from the attention's mass partials over those
     rows only. k = 1 uses every row.
+
+    ``overlap`` (default) runs step() on three streams of its own (a side
+    stream for the decisions and cache updates, two higher-priority streams
+    for the attentions), forked from and joined to the caller's stream per
+    step; the results equal the one-stream order bit for bit.
     """
 
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
