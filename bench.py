@@ -252,6 +252,21 @@ def make_inputs(wl, device):
     return inputs
 
 
+def union_length(intervals):
+    """Total length of the union of [start, end] intervals (overlaps counted once)."""
+    busy, cur_a, cur_b = 0.0, None, None
+    for a, b in sorted(intervals):
+        if cur_b is None or a > cur_b:
+            if cur_b is not None:
+                busy += cur_b - cur_a
+            cur_a, cur_b = a, b
+        else:
+            cur_b = max(cur_b, b)
+    if cur_b is not None:
+        busy += cur_b - cur_a
+    return busy
+
+
 def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False, clocks=None,
                     barrier=None, cue="product", theta=None, diagnostics=False, diag_row_stride=8):
     """Run warmup + timed steps (cycling the trajectory); returns timing dict."""
@@ -319,18 +334,7 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
             ms_sum += e0.elapsed_time(e1)
             iv.append((step_ev[0].elapsed_time(e0), step_ev[0].elapsed_time(e1)))
             flops += sum(attn_flops(wl, m) for m in modes[t, b])
-        iv.sort()
-        busy, cur_a, cur_b = 0.0, None, None
-        for a, b_ in iv:
-            if cur_b is None or a > cur_b:
-                if cur_b is not None:
-                    busy += cur_b - cur_a
-                cur_a, cur_b = a, b_
-            else:
-                cur_b = max(cur_b, b_)
-        if cur_b is not None:
-            busy += cur_b - cur_a
-        res["attn_ms"] = busy
+        res["attn_ms"] = union_length(iv)
         res["attn_ms_sum_of_launches"] = ms_sum
         res["attn_flops"] = flops
         res["attn_launches"] = len(ev)
