@@ -108,6 +108,8 @@ struct Tile {
   bool live;
 };
 
+constexpr int GROUP_M = 16;  // tile rows per band of the tile order
+
 template <int TM>  // output rows per tile: 128 (one CTA) or 256 (a CTA pair)
 __device__ __forceinline__ Tile decode(const Params& p, int64_t t) {
   Tile r;
@@ -119,8 +121,17 @@ __device__ __forceinline__ Tile decode(const Params& p, int64_t t) {
   r.seg = g;
   r.s = int(local / per_sample);
   const int64_t rem = local - int64_t(r.s) * per_sample;
-  r.m0 = int(rem / p.n_tiles_n) * TM;
-  r.n0 = int(rem % p.n_tiles_n) * BN;
+  // Grouped order: bands of GROUP_M tile rows, rows fastest inside a band, so
+  // the tiles in flight at once (one per CTA pair) share a few A row blocks
+  // and a few W column blocks that stay in L2, and W streams from HBM once per
+  // band instead of once per wave.
+  const int64_t band_tiles = int64_t(GROUP_M) * p.n_tiles_n;
+  const int band = int(rem / band_tiles);
+  const int m_first = band * GROUP_M;
+  const int rows = min(GROUP_M, sg.m_tiles - m_first);
+  const int idx = int(rem - int64_t(band) * band_tiles);
+  r.m0 = (m_first + idx % rows) * TM;
+  r.n0 = (idx / rows) * BN;
   r.live = true;
   if (sg.gated) {
     const int m = __ldg(p.mode + r.s);
