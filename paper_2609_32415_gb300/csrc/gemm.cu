@@ -7,9 +7,11 @@
 //
 // Two kernels: CTA pairs on 256 x 256 output tiles (gemm_pair_kernel, below,
 // used when a call has at least a wave of such tiles) and one CTA per SM on
-// 128 x 256 tiles (gemm_kernel), both persistent, K in 64-column steps. Tiles are numbered segment-major, then sample, then row tile, then
-// column tile (columns fastest, so the CTAs that run at once share A rows and
-// stream W through L2); CTA c takes tiles c, c + G, c + 2G, ...
+// 128 x 256 tiles (gemm_kernel), both persistent, K in 64-column steps. Tiles
+// are numbered segment-major, then sample, then in bands of GROUP_M row tiles,
+// rows fastest inside a band (so the CTAs that run at once share a few A row
+// blocks and a few W column blocks, both held in L2); CTA c takes tiles c,
+// c + G, c + 2G, ...
 //   warp 0      TMA producer: per K step one 128 x 64 A box and one 256 x 64 W
 //               box (128-byte swizzle, rows past a segment's end read as
 //               zeros) into a 4-stage ring.
