@@ -119,3 +119,17 @@ def test_host_validation_rejects_before_launch(lib):
     assert lib.refadapt_ref_cache_update(ctypes.byref(k), ctypes.byref(k), ctypes.byref(k), ctypes.byref(k),
                                          1, 1, 80, None, None, 0, 0, 0x70000, 0, None, None) == RA_EINVAL
     assert lib.refadapt_selftest_wait_timeout(None, 1000, None) == RA_EINVAL
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """With librefadapt.so absent every entry point raises; nothing falls back to
+    a CPU implementation."""
+    from paper_2609_32415_gb300 import _lib, api
+    monkeypatch.setattr(_lib, "LIB_PATH", str(tmp_path / "librefadapt.so"))
+    monkeypatch.setattr(_lib, "_lib", None)
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        _lib.load()
+    with pytest.raises(RuntimeError, match="missing"):
+        api.refadapt_mass_partial_len(256, 4096)
+    with pytest.raises(RuntimeError, match="missing"):
+        api.refadapt_state_size(1)
