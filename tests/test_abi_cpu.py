@@ -103,6 +103,14 @@ def test_host_validation_rejects_before_launch(lib):
     assert lib.refadapt_joint_attn(ctypes.byref(a), None) == RA_EINVAL
     a.q[2] = _seg(0x12000, 64, sn=100)   # stride not a multiple of 8 elements
     assert lib.refadapt_joint_attn(ctypes.byref(a), None) == RA_EINVAL
+    a.q[2] = _seg(0x12000, 64)
+    a.k[2] = a.v[2] = _seg(0x12000, 0)   # no target keys
+    assert lib.refadapt_joint_attn(ctypes.byref(a), None) == RA_EINVAL
+    assert b"at least one key row" in lib.refadapt_last_error()
+    q0 = _seg(0x10000, 0)
+    assert lib.refadapt_q_delta(ctypes.byref(q0), ctypes.byref(q0), 1, 1, 128, 1e-6, 0x30000, 0x40000,
+                                1 << 20, None) == RA_EINVAL   # empty slab: D undefined
+    assert b">= 1" in lib.refadapt_last_error()
     q1, q2 = _seg(0x10000, 10), _seg(0x20000, 11)
     assert lib.refadapt_q_delta(ctypes.byref(q1), ctypes.byref(q2), 1, 1, 128, 1e-6, 0x30000, 0x40000,
                                 1 << 20, None) == RA_EINVAL
