@@ -122,8 +122,11 @@ TILE_MODES = [1, 2]
 
 @pytest.mark.parametrize("tile_mode", TILE_MODES)
 @pytest.mark.parametrize("K,N,rows", [(64, 256, [1]), (256, 768, [40, 130, 77]), (3072, 512, [300]),
-                                      (512, 2048, [2500])])
+                                      (512, 2048, [2500]), (128, 512, [4500, 70])])
 def test_gemm_store_matches_oracle(cuda_ok, K, N, rows, tile_mode):
+    """Tiles are numbered in bands of 16 tile rows: 4500 rows make a full band
+    and a partial one of 256-row tiles (18 = 16 + 2) and of 128-row tiles
+    (36 = 16 + 16 + 4), followed by a second segment."""
     from paper_2609_32415_gb300._lib import RA_EPI_STORE
     _gemm_case(2, K, N, rows, RA_EPI_STORE, torch.Generator().manual_seed(K + N), tile_mode=tile_mode)
 
