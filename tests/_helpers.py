@@ -9,8 +9,10 @@ import oracle
 
 ROLES = ("text", "ref", "tgt")
 
-# Tolerances (BASELINE the benchmark spec): O max relative error 1e-2, M 1e-3 absolute,
-# D 1e-4 relative; gate modes exact except |gbar - theta| < 1e-4.
+# Parity tolerances of the hot path against the fp64 oracle: O max relative
+# error 1e-2 (bf16 P and O round at 2^-9 relative), M 1e-3 absolute, D 1e-4
+# relative; gate modes exact except where |gbar - theta| < 1e-4, where the
+# GPU's fp32 score and the oracle's fp64 score may fall on either side.
 O_REL = 1e-2
 M_ABS = 1e-3
 D_REL = 1e-4
