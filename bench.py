@@ -745,7 +745,8 @@ def main_ours(args):
         "roofline": {"bound": "tensor", "kernel": "joint_attn_kernel<128>",
                      "achieved": round(attn_tflops, 1), "peak": peaks["bf16_sustained"],
                      "unit": "TFLOP/s", "frac": round(attn_tflops / peaks["bf16_sustained"], 4),
-                     "traffic": traffic,
+                     "traffic": None if traffic is None else traffic["bytes"],
+                     "traffic_capture": traffic,
                      "flops_per_launch": int(per_launch_flops),
                      "launch_ms": round(main["attn_ms"] / main["attn_launches"], 4),
                      "peak_kind": "%s, sustained bf16 (kernel timed inside a long step)" % peaks["source"]},
