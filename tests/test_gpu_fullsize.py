@@ -57,13 +57,21 @@ def _run_stack(wl, blocks):
     return sub, rec
 
 
-@pytest.mark.parametrize("name", ["c2", "c3", "c4"])
-def test_fullsize_block_parity(cuda_ok, name):
+FULLSIZE = [("c2", {}), ("c3", {}), ("c4", {}),
+            # sweep points: 64k tokens, 90 % reference, boundary forced at block 4
+            # (block 0 reuses at step 1); 8k tokens, 50 % reference, boundary at block 7
+            ("c5", dict(total=65536, ref_frac=0.9, reuse_frac=0.5)),
+            ("c5", dict(total=8192, ref_frac=0.5, reuse_frac=0.9))]
+
+
+@pytest.mark.parametrize("name,over", FULLSIZE,
+                         ids=["c2", "c3", "c4", "sweep-64k-90ref-50reuse", "sweep-8k-50ref-90reuse"])
+def test_fullsize_block_parity(cuda_ok, name, over):
     """First block of the stack, steps 0 and 1: sampled O rows of every
     executed role, two mass tiles per sampled head, D of every head, and the
     step-1 decision from the oracle controller with the oracle's D."""
     from paper_2609_32415_gb300 import synth
-    wl = synth.make_workload(name)
+    wl = synth.make_workload(name, **over)
     wl.n_steps = 2
     sub, rec = _run_stack(wl, [0])
     sc = 1.0 / math.sqrt(sub.d)
