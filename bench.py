@@ -769,7 +769,8 @@ def main_ours(args):
         if graph.get("error"):
             line["cuda_graph_error"] = graph["error"]
         elif "modes" in graph:
-            line["cuda_graph_modes_match"] = bool((graph["modes"] == main["modes"]).all())
+            timed = sorted(set(main["steps_t"]))   # steps both runs executed
+            line["cuda_graph_modes_match"] = bool((graph["modes"][timed] == main["modes"][timed]).all())
     if refresh is not None:
         rms = refresh["total_ms"] / args.steps
         line["always_refresh_ms_per_step"] = round(rms, 3)
