@@ -550,20 +550,16 @@ def time_e2e(wl, inputs, warmup, steps):
                         "the mean over the timed steps"}
 
 
-def time_q_delta(wl, inputs, reps=64):
-    """HBM roofline of the Q-change reduction alone: target Q of step 1 vs step
-    0, rotating over 8 blocks (8 x 50 MB > L2, so every launch reads HBM).
-    The launches are queued behind a GPU-side sleep so they run back to back;
-    the average launch duration is the events' span divided by the launches."""
+def _q_delta_launch_ms(pairs, B, H, eps, reps):
+    """Average duration of one refadapt_q_delta launch over `reps` launches
+    rotating over `pairs` (current, previous), queued behind a GPU-side sleep
+    so they run back to back; the best of three runs."""
     import torch
-    from paper_2609_32415_gb300 import api, roles_from_joint
-    nb = min(8, wl.n_blocks)
-    pairs = [(roles_from_joint(inputs[1][b], wl.offsets(), wl.n)["tgt"][0],
-              roles_from_joint(inputs[0][b], wl.offsets(), wl.n)["tgt"][0]) for b in range(nb)]
-    ws = api.q_delta_workspace(wl.B, wl.H)
-    out = torch.empty((wl.B, wl.H), dtype=torch.float32, device="cuda")
-    for i in range(nb):                          # warm-up
-        api.refadapt_q_delta(pairs[i][0], pairs[i][1], out, ws, wl.eps)
+    from paper_2609_32415_gb300 import api
+    ws = api.q_delta_workspace(B, H)
+    out = torch.empty((B, H), dtype=torch.float32, device="cuda")
+    for a, b in pairs:                           # warm-up
+        api.refadapt_q_delta(a, b, out, ws, eps)
     runs = []
     for _ in range(3):
         torch.cuda.synchronize()
@@ -571,13 +567,45 @@ def time_q_delta(wl, inputs, reps=64):
         torch.cuda._sleep(20_000_000)            # ~10 ms: the host queues every launch meanwhile
         e0.record()
         for i in range(reps):
-            a, b = pairs[i % nb]
-            api.refadapt_q_delta(a, b, out, ws, wl.eps)
+            a, b = pairs[i % len(pairs)]
+            api.refadapt_q_delta(a, b, out, ws, eps)
         e1.record()
         torch.cuda.synchronize()
         runs.append(e0.elapsed_time(e1) / reps)
+    return min(runs)
+
+
+def time_q_delta_long(n_tgt=16380, H=24, d=128, eps=1e-6, reps=64):
+    """The same kernel on a longer read: the video workload's target-query
+    shape (16,380 rows; 2 x 100.6 MB per launch), four rotating seeded pairs
+    (805 MB > L2)."""
+    import torch
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0x5EED)
+    pairs = []
+    for _ in range(4):
+        prev = (torch.randn((1, H, n_tgt, d), generator=g, device="cuda") / d ** 0.5).to(torch.bfloat16)
+        cur = (prev.float() + 0.4 * torch.randn((1, H, n_tgt, d), generator=g, device="cuda") / d ** 0.5
+               ).to(torch.bfloat16)
+        pairs.append((cur, prev))
+    ms = _q_delta_launch_ms(pairs, 1, H, eps, reps)
+    byts = 4 * n_tgt * H * d
+    del pairs
+    return {"bytes": byts, "ms": ms, "gbs": byts / ms / 1e6}
+
+
+def time_q_delta(wl, inputs, reps=64):
+    """HBM roofline of the Q-change reduction alone: target Q of step 1 vs step
+    0, rotating over 8 blocks (8 x 50 MB > L2, so every launch reads HBM).
+    The launches are queued behind a GPU-side sleep so they run back to back;
+    the average launch duration is the events' span divided by the launches."""
+    import torch
+    from paper_2609_32415_gb300 import roles_from_joint
+    nb = min(8, wl.n_blocks)
+    pairs = [(roles_from_joint(inputs[1][b], wl.offsets(), wl.n)["tgt"][0],
+              roles_from_joint(inputs[0][b], wl.offsets(), wl.n)["tgt"][0]) for b in range(nb)]
+    ms = _q_delta_launch_ms(pairs, wl.B, wl.H, wl.eps, reps)
     byts = 4 * wl.n_tgt * wl.H * wl.d * wl.B
-    ms = min(runs)
     # Context: a library streaming read of the same number of bytes (torch's
     # sum over one contiguous buffer), timed the same way.
     bufs = [torch.ones(byts // 2, dtype=torch.bfloat16, device="cuda") for _ in range(8)]
@@ -666,6 +694,7 @@ def main_ours(args):
     if not args.no_refresh_baseline:
         refresh = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1, barrier=barrier)
     qd = time_q_delta(wl, inputs)
+    qd_long = time_q_delta_long(H=wl.H, d=wl.d, eps=wl.eps) if wl.d == 128 else None
     diag = None
     if args.diagnostics:
         diag = time_trajectory(wl, inputs, args.warmup, args.steps, diagnostics=True, diag_row_stride=8)
@@ -754,7 +783,12 @@ def main_ours(args):
                              "unit": "GB/s", "frac": round(qd["gbs"] / peaks["hbm_gbs"], 4),
                              "bytes_per_launch": qd["bytes"], "launch_ms": round(qd["ms"], 5),
                              "same_bytes_torch_sum_gbs": round(qd["lib_read_gbs"], 1),
-                             "peak_kind": "%s HBM copy" % peaks["source"]},
+                             "peak_kind": "%s HBM copy" % peaks["source"],
+                             "longer_read": None if qd_long is None else {
+                                 "shape": "video target query, 16,380 rows x %d heads x d %d" % (wl.H, wl.d),
+                                 "bytes_per_launch": qd_long["bytes"], "launch_ms": round(qd_long["ms"], 5),
+                                 "achieved": round(qd_long["gbs"], 1),
+                                 "frac": round(qd_long["gbs"] / peaks["hbm_gbs"], 4)}},
         "gpu_launches": main["launches"],
         "clocks": main["clocks"],
         "e2e": e2e,
