@@ -61,15 +61,18 @@ FULLSIZE = [("c2", {}), ("c3", {}), ("c4", {}),
             # sweep points: 64k tokens, 90 % reference, boundary forced at block 4
             # (block 0 reuses at step 1); 8k tokens, 50 % reference, boundary at block 7
             ("c5", dict(total=65536, ref_frac=0.9, reuse_frac=0.5)),
-            ("c5", dict(total=8192, ref_frac=0.5, reuse_frac=0.9))]
+            ("c5", dict(total=8192, ref_frac=0.5, reuse_frac=0.9)),
+            # two samples: per-sample strides and the grid's sample dimension at scale
+            ("c5", dict(total=16384, ref_frac=0.7, reuse_frac=0.5, B=2))]
 
 
 @pytest.mark.parametrize("name,over", FULLSIZE,
-                         ids=["c2", "c3", "c4", "sweep-64k-90ref-50reuse", "sweep-8k-50ref-90reuse"])
+                         ids=["c2", "c3", "c4", "sweep-64k-90ref-50reuse", "sweep-8k-50ref-90reuse",
+                              "sweep-16k-70ref-50reuse-B2"])
 def test_fullsize_block_parity(cuda_ok, name, over):
-    """First block of the stack, steps 0 and 1: sampled O rows of every
-    executed role, two mass tiles per sampled head, D of every head, and the
-    step-1 decision from the oracle controller with the oracle's D."""
+    """First block of the stack, steps 0 and 1, every sample: sampled O rows
+    of every executed role, two mass tiles per sampled head, D of every head,
+    and the step-1 decisions from the oracle controller with the oracle's D."""
     from paper_2609_32415_gb300 import synth
     wl = synth.make_workload(name, **over)
     wl.n_steps = 2
@@ -78,65 +81,68 @@ def test_fullsize_block_parity(cuda_ok, name, over):
     bias = None if sub.bias is None else np.asarray(sub.bias)
     rng = np.random.default_rng(0)
     a_b = 0                                    # the cache holds step 0 after step 0's FULL
+    hs = list(HEADS)
+    r0, r1 = sub.n_text, sub.n_text + sub.n_ref
     for t in range(2):
         r = rec[(t, 0)]
-        mode = int(r["mode"][0])
-        if t == 0:
-            assert mode == 3
         X = r["X"]
-        fresh_ref = mode in (2, 3)
-        Xk = X if fresh_ref else rec[(a_b, 0)]["X"]
-        hs = list(HEADS)
-        q = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 0)[0, hs]) for ro in ROLES}
-        k = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 1)[0, hs]) for ro in ROLES}
-        v = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 2)[0, hs]) for ro in ROLES}
-        keys = np.concatenate([k["text"], k["ref"], k["tgt"]], axis=1)
-        vals = np.concatenate([v["text"], v["ref"], v["tgt"]], axis=1)
-        r0, r1 = sub.n_text, sub.n_text + sub.n_ref
-        roles = ("text", "tgt") if mode == 0 else ROLES
-        for ro in roles:
-            n = sub.n[ro]
-            idx = np.unique(np.concatenate([np.arange(min(8, n)), np.arange(max(0, n - 8), n),
-                                            rng.choice(n, size=min(48, n), replace=False)]))
-            rb = np.full(len(idx), 1 if ro == "tgt" else 0, dtype=np.uint8)
-            o, _ = oracle.joint_attention(q[ro][:, idx], keys, vals, sc,
-                                          None if bias is None else bias[hs], rb if bias is not None else None,
-                                          (r0, r1))
-            got = r["O"][ro][0, hs][:, idx].double().cpu().numpy()
-            ok, worst, nw = o_close(got, o)
-            assert ok, (name, t, ro, worst, nw)
-        if mode == 0:
-            assert torch.isnan(r["O"]["ref"].float()).all()
-        # mass partials: first and last target tile of the sampled heads
-        nt = (sub.n_tgt + 127) // 128
-        base = (sub.n_text + 127) // 128
-        for tile in (0, nt - 1):
-            rows = np.arange(tile * 128, min(sub.n_tgt, tile * 128 + 128))
-            rb = np.ones(len(rows), dtype=np.uint8)
-            _, m = oracle.joint_attention(q["tgt"][:, rows], keys, vals, sc,
-                                          None if bias is None else bias[hs], rb if bias is not None else None,
-                                          (r0, r1), want_o=False)
-            got = r["mass"][0, hs, base + tile].double().cpu().numpy() / len(rows)
-            err = np.abs(got - m.mean(axis=1)).max()
-            assert err <= M_ABS, (name, t, tile, err)
-            assert err <= 2e-5, (name, t, tile, err)   # far below the gate's 1e-4 band
+        for z in range(sub.B):
+            mode = int(r["mode"][z])
+            if t == 0:
+                assert mode == 3
+            fresh_ref = mode in (2, 3)
+            Xk = X if fresh_ref else rec[(a_b, 0)]["X"]
+            q = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 0)[z, hs]) for ro in ROLES}
+            k = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 1)[z, hs]) for ro in ROLES}
+            v = {ro: _wide(_role(X if ro != "ref" else Xk, sub, ro, 2)[z, hs]) for ro in ROLES}
+            keys = np.concatenate([k["text"], k["ref"], k["tgt"]], axis=1)
+            vals = np.concatenate([v["text"], v["ref"], v["tgt"]], axis=1)
+            roles = ("text", "tgt") if mode == 0 else ROLES
+            for ro in roles:
+                n = sub.n[ro]
+                idx = np.unique(np.concatenate([np.arange(min(8, n)), np.arange(max(0, n - 8), n),
+                                                rng.choice(n, size=min(48, n), replace=False)]))
+                rb = np.full(len(idx), 1 if ro == "tgt" else 0, dtype=np.uint8)
+                o, _ = oracle.joint_attention(q[ro][:, idx], keys, vals, sc,
+                                              None if bias is None else bias[hs],
+                                              rb if bias is not None else None, (r0, r1))
+                got = r["O"][ro][z, hs][:, idx].double().cpu().numpy()
+                ok, worst, nw = o_close(got, o)
+                assert ok, (name, t, z, ro, worst, nw)
+            if mode == 0:
+                assert torch.isnan(r["O"]["ref"][z].float()).all()
+            # mass partials: first and last target tile of the sampled heads
+            nt = (sub.n_tgt + 127) // 128
+            base = (sub.n_text + 127) // 128
+            for tile in (0, nt - 1):
+                rows = np.arange(tile * 128, min(sub.n_tgt, tile * 128 + 128))
+                rb = np.ones(len(rows), dtype=np.uint8)
+                _, m = oracle.joint_attention(q["tgt"][:, rows], keys, vals, sc,
+                                              None if bias is None else bias[hs],
+                                              rb if bias is not None else None, (r0, r1), want_o=False)
+                got = r["mass"][z, hs, base + tile].double().cpu().numpy() / len(rows)
+                err = np.abs(got - m.mean(axis=1)).max()
+                assert err <= M_ABS, (name, t, z, tile, err)
+                assert err <= 2e-5, (name, t, z, tile, err)   # far below the gate's 1e-4 band
         if t == 1:
-            qc = _wide(_role(X, sub, "tgt", 0)[0])
-            qp = _wide(_role(r["Xprev"], sub, "tgt", 0)[0])
-            D = oracle.q_change(qc, qp, sub.eps)
-            got = r["D"][0].double().cpu().numpy()
+            qc = _wide(_role(X, sub, "tgt", 0))
+            qp = _wide(_role(r["Xprev"], sub, "tgt", 0))
+            D = oracle.q_change(qc, qp, sub.eps)                       # [B, H]
+            got = r["D"].double().cpu().numpy()
             assert (np.abs(got - D) / D).max() <= D_REL
-            # the controller's decision from the oracle D and the mass of step 0
+            # the controller's decisions from the oracle D and the mass of step 0
             # (the GPU's M, whose sampled tiles were checked above at step 0)
-            M_prev = rec[(0, 0)]["mass"][0].double().sum(-1).cpu().numpy() / sub.n_tgt
-            gate = oracle.Gate(1, sub.theta, sub.delta_max, sub.forced_boundary)
+            M_prev = rec[(0, 0)]["mass"].double().sum(-1).cpu().numpy() / sub.n_tgt
+            gate = oracle.Gate(sub.B, sub.theta, sub.delta_max, sub.forced_boundary)
             gate.begin_step(0)
             gate.decide(0, 0)
             gate.begin_step(1)
-            modes, gbar = gate.decide(1, 0, D[None], M_prev[None],
-                                      tie=lambda tt, bb, s: mode == 1, tie_band=TIE_BAND)
-            assert modes[0] == mode, (name, modes, mode, gbar, sub.theta)
-            assert abs(gbar[0] - float(r["gbar"][0])) < 1e-5 * max(1.0, abs(gbar[0]))
+            gpu_modes = [int(x) for x in r["mode"]]
+            modes, gbar = gate.decide(1, 0, D, M_prev,
+                                      tie=lambda tt, bb, s: gpu_modes[s] == 1, tie_band=TIE_BAND)
+            assert modes == gpu_modes, (name, modes, gpu_modes, gbar, sub.theta)
+            for z in range(sub.B):
+                assert abs(gbar[z] - float(r["gbar"][z])) < 1e-5 * max(1.0, abs(gbar[z]))
 
 
 def test_fullsize_depth_reduced_trajectory(cuda_ok):
