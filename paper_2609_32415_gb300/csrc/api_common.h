@@ -17,6 +17,12 @@ void clear_error();
 uint64_t wait_budget_ns();
 int num_sms();  // of the current device (cached per device)
 
+// Raises `func`'s dynamic shared-memory limit to `bytes` on the current
+// device, once per (function, device): the attribute belongs to the device's
+// context, so a process that drives several GPUs sets it on each. Returns
+// RA_ECUDA with the reason recorded (prefixed by `who`) on failure.
+ra_status ensure_dynamic_smem(const void* func, int bytes, const char* who);
+
 // A bf16 segment usable by 16-byte vector access and by TMA: 16-byte aligned
 // pointer and strides, n >= 0, non-negative strides. `what` names it in errors.
 bool check_seg(const ra_seg& s, const char* what, bool allow_null_if_empty = true);

@@ -7,6 +7,7 @@
 #include <cstdarg>
 #include <cstdio>
 #include <mutex>
+#include <vector>
 
 #include "api_common.h"
 #include "tc_ptx.cuh"
@@ -29,6 +30,34 @@ void set_error(const char* fmt, ...) {
 void clear_error() { g_err[0] = 0; }
 
 uint64_t wait_budget_ns() { return g_budget_ns.load(std::memory_order_relaxed); }
+
+namespace {
+struct SmemAttrKey {
+  const void* func;
+  int dev;
+};
+std::mutex g_smem_attr_mu;
+std::vector<SmemAttrKey> g_smem_attr_done;
+}  // namespace
+
+ra_status ensure_dynamic_smem(const void* func, int bytes, const char* who) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    set_error("%s: cudaGetDevice: %s", who, cudaGetErrorString(e));
+    return RA_ECUDA;
+  }
+  std::lock_guard<std::mutex> lk(g_smem_attr_mu);
+  for (const SmemAttrKey& k : g_smem_attr_done)
+    if (k.func == func && k.dev == dev) return RA_OK;
+  e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+  if (e != cudaSuccess) {
+    set_error("%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
+    return RA_ECUDA;
+  }
+  g_smem_attr_done.push_back({func, dev});
+  return RA_OK;
+}
 
 int num_sms() {
   int dev = 0;

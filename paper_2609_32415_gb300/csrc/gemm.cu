@@ -713,17 +713,10 @@ extern "C" ra_status refadapt_gemm(const ra_gemm_args* a, void* stream) {
   }
   p.total_tiles = tiles;
   if (tiles == 0) return RA_OK;
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_ALLOC);
-    if (attr_err == cudaSuccess)
-      attr_err = cudaFuncSetAttribute(gemm_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, P_SMEM_ALLOC);
-  });
-  if (attr_err != cudaSuccess) {
-    set_error("refadapt_gemm: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
-    return RA_ECUDA;
-  }
+  ra_status as = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_kernel), SMEM_ALLOC, "refadapt_gemm");
+  if (as == RA_OK)
+    as = ensure_dynamic_smem(reinterpret_cast<const void*>(gemm_pair_kernel), P_SMEM_ALLOC, "refadapt_gemm");
+  if (as != RA_OK) return as;
   const cudaStream_t st = static_cast<cudaStream_t>(stream);
   if (!pair) {
     const int64_t grid = tiles < sms ? tiles : sms;

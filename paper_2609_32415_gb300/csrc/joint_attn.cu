@@ -492,16 +492,9 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
 // ------------------------------------------------------------------ host side
 template <int D>
 ra_status launch(const Params& p, dim3 grid, cudaStream_t st) {
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(joint_attn_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    Cfg<D>::SMEM_ALLOC);
-  });
-  if (attr_err != cudaSuccess) {
-    set_error("refadapt_joint_attn: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
-    return RA_ECUDA;
-  }
+  const ra_status as = ensure_dynamic_smem(reinterpret_cast<const void*>(joint_attn_kernel<D>), Cfg<D>::SMEM_ALLOC,
+                                           "refadapt_joint_attn");
+  if (as != RA_OK) return as;
   joint_attn_kernel<D><<<grid, NUM_THREADS, Cfg<D>::SMEM_ALLOC, st>>>(p);
   return launch_status("refadapt_joint_attn");
 }

@@ -638,15 +638,9 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
              !encode_seg(&p.tm_p, *q_prev, B, H, d, d, p.rows_per_unit, false)) {
     return RA_EINVAL;
   }
-  static std::once_flag once;
-  static cudaError_t attr_err = cudaSuccess;
-  std::call_once(once, [] {
-    attr_err = cudaFuncSetAttribute(qd::q_delta_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, qd::SMEM_ALLOC);
-  });
-  if (attr_err != cudaSuccess) {
-    set_error("refadapt_q_delta: cudaFuncSetAttribute: %s", cudaGetErrorString(attr_err));
-    return RA_ECUDA;
-  }
+  const ra_status as = ensure_dynamic_smem(reinterpret_cast<const void*>(qd::q_delta_kernel), qd::SMEM_ALLOC,
+                                           "refadapt_q_delta");
+  if (as != RA_OK) return as;
   qd::q_delta_kernel<<<p.grid, qd::THREADS, qd::SMEM_ALLOC, static_cast<cudaStream_t>(stream)>>>(p);
   return launch_status("refadapt_q_delta");
 }
