@@ -19,6 +19,11 @@
  *    time budget sets bit 0 of the caller's error word (see
  *    refadapt_check_error), never traps, and leaves the context usable.
  *  - No exceptions cross the ABI; nothing calls exit().
+ *  - Calls may come from several host threads and target several GPUs: each
+ *    works on the device current in the calling thread, and the library's
+ *    one-time set-up (kernel shared-memory limits, SM counts, cluster
+ *    occupancy, the no-allocation scratch address) is kept per device under
+ *    a mutex. Work on one device follows the stream order the caller gives.
  *  - bf16 tensors are described by ra_seg: element (b, h, n, c) lives at
  *    ptr + b*stride_b + h*stride_h + n*stride_n + c (strides in elements,
  *    c contiguous). ptr and every stride must be 16-byte aligned

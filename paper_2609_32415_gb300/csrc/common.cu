@@ -7,7 +7,6 @@
 #include <cstdarg>
 #include <cstdio>
 #include <mutex>
-#include <vector>
 
 #include "api_common.h"
 #include "tc_ptx.cuh"
@@ -36,8 +35,12 @@ struct SmemAttrKey {
   const void* func;
   int dev;
 };
+// Fixed-size record (no allocation, nothing that can throw across the ABI);
+// past its capacity the attribute is simply set again on every call.
+constexpr int kSmemAttrSlots = 256;
 std::mutex g_smem_attr_mu;
-std::vector<SmemAttrKey> g_smem_attr_done;
+SmemAttrKey g_smem_attr_done[kSmemAttrSlots];
+int g_smem_attr_count = 0;
 }  // namespace
 
 ra_status ensure_dynamic_smem(const void* func, int bytes, const char* who) {
@@ -48,14 +51,14 @@ ra_status ensure_dynamic_smem(const void* func, int bytes, const char* who) {
     return RA_ECUDA;
   }
   std::lock_guard<std::mutex> lk(g_smem_attr_mu);
-  for (const SmemAttrKey& k : g_smem_attr_done)
-    if (k.func == func && k.dev == dev) return RA_OK;
+  for (int i = 0; i < g_smem_attr_count; ++i)
+    if (g_smem_attr_done[i].func == func && g_smem_attr_done[i].dev == dev) return RA_OK;
   e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
   if (e != cudaSuccess) {
     set_error("%s: cudaFuncSetAttribute: %s", who, cudaGetErrorString(e));
     return RA_ECUDA;
   }
-  g_smem_attr_done.push_back({func, dev});
+  if (g_smem_attr_count < kSmemAttrSlots) g_smem_attr_done[g_smem_attr_count++] = {func, dev};
   return RA_OK;
 }
 
