@@ -22,8 +22,9 @@
  *  - Calls may come from several host threads and target several GPUs: each
  *    works on the device current in the calling thread, and the library's
  *    one-time set-up (kernel shared-memory limits, SM counts, cluster
- *    occupancy, the no-allocation scratch address) is kept per device under
- *    a mutex. Work on one device follows the stream order the caller gives.
+ *    occupancy) is kept per device under a mutex, the no-allocation scratch
+ *    address per device and CUDA context. Work on one device follows the
+ *    stream order the caller gives.
  *  - bf16 tensors are described by ra_seg: element (b, h, n, c) lives at
  *    ptr + b*stride_b + h*stride_h + n*stride_n + c (strides in elements,
  *    c contiguous). ptr and every stride must be 16-byte aligned
@@ -184,12 +185,17 @@ ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B,
  * the library holds it until the process exits. Larger B * H returns RA_EINVAL
  * (use refadapt_q_delta with a workspace). The call allocates nothing: no
  * cudaMalloc, no cudaFree, no allocating library routine. Its first call on a
- * device looks the array's device address up once (cudaGetSymbolAddress with
- * that device current) and caches it; make that first call before any stream
- * capture. Every call clears the counters on `stream` before its kernel; all
- * calls share the one array, so calls that overlap on the GPU (different
- * streams, or different host threads without ordering) race and must not be
- * issued. Arguments and results are those of refadapt_q_delta.
+ * device looks the array's device address up (cudaGetSymbolAddress with that
+ * device current) and caches it for the CUDA context current at that moment;
+ * a later call in another context (for instance after cudaDeviceReset tore
+ * the primary context down) looks it up again. Make the first call, and the
+ * first call after a reset, before any stream capture. A call that takes the
+ * multi-block path clears that path's ticket counters on `stream` right
+ * before its kernel, after every argument check; a call that returns
+ * RA_EINVAL queues nothing. All calls share the one array, so calls that
+ * overlap on the GPU (different streams, or different host threads without
+ * ordering) race and must not be issued. Arguments and results are those of
+ * refadapt_q_delta.
  */
 #define RA_Q_DELTA_NOALLOC_MAX_BH 96
 ra_status refadapt_q_delta_noalloc(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,

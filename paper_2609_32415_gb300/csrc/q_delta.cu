@@ -482,38 +482,48 @@ extern "C" size_t refadapt_q_delta_workspace_size(int32_t B, int32_t H) {
   return counters + bh * ra::qd::MAX_SPLITS * 2 * sizeof(double);
 }
 
-extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
-                                      float eps, float* d_out, void* workspace, size_t workspace_bytes,
-                                      void* stream) {
-  using namespace ra;
-  clear_error();
-  if (!q_cur || !q_prev || !d_out || !workspace) {
-    set_error("refadapt_q_delta: NULL argument");
+namespace ra {
+namespace qd {
+
+// Argument checks shared by both entry points (everything but the workspace).
+ra_status validate(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
+                   float eps, const float* d_out) {
+  if (!q_cur || !q_prev || !d_out) {
+    set_error("%s: NULL argument", who);
     return RA_EINVAL;
   }
   if (d != 64 && d != 128) {
-    set_error("refadapt_q_delta: d = %d (supported: 64, 128)", d);
+    set_error("%s: d = %d (supported: 64, 128)", who, d);
     return RA_EINVAL;
   }
   if (B < 1 || H < 1 || B > 65535 || H > 65535) {
-    set_error("refadapt_q_delta: B = %d, H = %d out of range", B, H);
+    set_error("%s: B = %d, H = %d out of range", who, B, H);
     return RA_EINVAL;
   }
-  if (!check_seg(*q_cur, "refadapt_q_delta: q_cur", false) || !check_seg(*q_prev, "refadapt_q_delta: q_prev", false))
-    return RA_EINVAL;
+  if (!check_seg(*q_cur, who, false) || !check_seg(*q_prev, who, false)) return RA_EINVAL;
   if (q_cur->n != q_prev->n || q_cur->n < 1) {
-    set_error("refadapt_q_delta: q_cur.n = %d and q_prev.n = %d must be equal and >= 1", q_cur->n, q_prev->n);
+    set_error("%s: q_cur.n = %d and q_prev.n = %d must be equal and >= 1", who, q_cur->n, q_prev->n);
     return RA_EINVAL;
   }
   if (!(eps >= 0.f)) {
-    set_error("refadapt_q_delta: eps must be >= 0");
+    set_error("%s: eps must be >= 0", who);
     return RA_EINVAL;
   }
-  if (reinterpret_cast<uintptr_t>(workspace) % 16 != 0 || workspace_bytes < refadapt_q_delta_workspace_size(B, H)) {
-    set_error("refadapt_q_delta: workspace must be 16-byte aligned and >= %zu bytes",
-              refadapt_q_delta_workspace_size(B, H));
+  const int rows_per_unit = UNIT_BYTES / (2 * d);
+  const int64_t units = int64_t(B) * H * ((q_cur->n + rows_per_unit - 1) / rows_per_unit);
+  if (units > (int64_t(1) << 30)) {
+    set_error("%s: problem too large", who);
     return RA_EINVAL;
   }
+  return RA_OK;
+}
+
+// Picks the cluster path or the multi-block path and launches it, after
+// validate(). The workspace is touched only by the multi-block path; with
+// clear_counters its ticket counters are zeroed on the stream right before
+// that kernel (for a workspace whose earlier contents are unknown).
+ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
+                 float eps, float* d_out, void* workspace, bool clear_counters, void* stream) {
   const int n = q_cur->n;
   const int bh = B * H;
   {
@@ -524,15 +534,15 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
     // run in one wave are candidates. Among those the one with the most bytes
     // in flight (CTAs x stages) wins. Taken when it occupies at least 60 % of
     // the CTAs the multi-block path would run (min(SMs, units)).
-    const int rows_per_unit = qd::UNIT_BYTES / (2 * d);
+    const int rows_per_unit = UNIT_BYTES / (2 * d);
     const int per_slab = (n + rows_per_unit - 1) / rows_per_unit;
     const int64_t sms = num_sms();
     int best_s = 0, best_cs = 0;
     int64_t best_score = 0;
     for (int S : {8, 4}) {
-      for (int cs = 1; cs <= qd::CL_MAX_CS && cs <= per_slab; ++cs) {
-        if ((per_slab + cs - 1) / cs > qd::CL_MAX_UNITS) continue;
-        const int fit = qd::max_active_clusters(S, cs);
+      for (int cs = 1; cs <= CL_MAX_CS && cs <= per_slab; ++cs) {
+        if ((per_slab + cs - 1) / cs > CL_MAX_UNITS) continue;
+        const int fit = max_active_clusters(S, cs);
         if (fit < 0) return RA_ECUDA;
         if (bh > fit) continue;
         const int64_t score = int64_t(bh) * cs * S;
@@ -546,7 +556,7 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
     const int64_t units_all = int64_t(bh) * per_slab;
     const int64_t ticket_ctas = units_all < sms ? units_all : sms;
     if (best_s != 0 && double(bh) * best_cs >= 0.6 * double(ticket_ctas)) {
-      qd::ClusterParams c;
+      ClusterParams c;
       std::memset(&c, 0, sizeof(c));
       c.bulk = (q_cur->stride_n == d && q_prev->stride_n == d) ? 1 : 0;
       c.base_c = static_cast<const char*>(q_cur->ptr);
@@ -570,8 +580,8 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
       cudaLaunchConfig_t cfg;
       std::memset(&cfg, 0, sizeof(cfg));
       cfg.gridDim = dim3(best_cs, H, B);
-      cfg.blockDim = dim3(best_s == 8 ? qd::ClLayout<8>::THREADS : qd::ClLayout<4>::THREADS, 1, 1);
-      cfg.dynamicSmemBytes = best_s == 8 ? qd::ClLayout<8>::ALLOC : qd::ClLayout<4>::ALLOC;
+      cfg.blockDim = dim3(best_s == 8 ? ClLayout<8>::THREADS : ClLayout<4>::THREADS, 1, 1);
+      cfg.dynamicSmemBytes = best_s == 8 ? ClLayout<8>::ALLOC : ClLayout<4>::ALLOC;
       cfg.stream = static_cast<cudaStream_t>(stream);
       cudaLaunchAttribute attr[2];
       attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -584,35 +594,31 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
       attr[1].val.programmaticStreamSerializationAllowed = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 2;
-      const cudaError_t e = best_s == 8 ? cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel<8>, c)
-                                        : cudaLaunchKernelEx(&cfg, qd::q_delta_cluster_kernel<4>, c);
+      const cudaError_t e = best_s == 8 ? cudaLaunchKernelEx(&cfg, q_delta_cluster_kernel<8>, c)
+                                        : cudaLaunchKernelEx(&cfg, q_delta_cluster_kernel<4>, c);
       if (e != cudaSuccess) {
-        set_error("refadapt_q_delta: cluster launch failed: %s", cudaGetErrorString(e));
+        set_error("%s: cluster launch failed: %s", who, cudaGetErrorString(e));
         cudaGetLastError();
         return RA_ECUDA;
       }
-      return launch_status("refadapt_q_delta");
+      return launch_status(who);
     }
   }
-  qd::Params p;
+  Params p;
   p.H = H;
-  p.rows_per_unit = qd::UNIT_BYTES / (2 * d);
+  p.rows_per_unit = UNIT_BYTES / (2 * d);
   p.per_slab = (n + p.rows_per_unit - 1) / p.rows_per_unit;
   const int64_t units = int64_t(bh) * p.per_slab;
-  if (units > (int64_t(1) << 30)) {
-    set_error("refadapt_q_delta: problem too large");
-    return RA_EINVAL;
-  }
   p.units = int(units);
   // One CTA per SM; at most MAX_SPLITS - 1 CTAs may share a slab (slots) and
   // at most MAX_UNITS_PER_CTA units may fall to one CTA.
   int64_t G = num_sms();
   if (G > units) G = units;
-  if (G > int64_t(qd::MAX_SPLITS - 1) * bh) G = int64_t(qd::MAX_SPLITS - 1) * bh;
-  while ((units + G - 1) / G > qd::MAX_UNITS_PER_CTA) G *= 2;
+  if (G > int64_t(MAX_SPLITS - 1) * bh) G = int64_t(MAX_SPLITS - 1) * bh;
+  while ((units + G - 1) / G > MAX_UNITS_PER_CTA) G *= 2;
   if (G > units) G = units;
-  if (G > int64_t(qd::MAX_SPLITS - 1) * bh || G > 2147483647) {
-    set_error("refadapt_q_delta: n = %d rows per slab is too large", n);
+  if (G > int64_t(MAX_SPLITS - 1) * bh || G > 2147483647) {
+    set_error("%s: n = %d rows per slab is too large", who, n);
     return RA_EINVAL;
   }
   p.grid = int(G);
@@ -638,18 +644,46 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
              !encode_seg(&p.tm_p, *q_prev, B, H, d, d, p.rows_per_unit, false)) {
     return RA_EINVAL;
   }
-  const ra_status as = ensure_dynamic_smem(reinterpret_cast<const void*>(qd::q_delta_kernel), qd::SMEM_ALLOC,
-                                           "refadapt_q_delta");
+  const ra_status as = ensure_dynamic_smem(reinterpret_cast<const void*>(q_delta_kernel), SMEM_ALLOC, who);
   if (as != RA_OK) return as;
-  qd::q_delta_kernel<<<p.grid, qd::THREADS, qd::SMEM_ALLOC, static_cast<cudaStream_t>(stream)>>>(p);
-  return launch_status("refadapt_q_delta");
+  if (clear_counters) {
+    const cudaError_t e = cudaMemsetAsync(workspace, 0, counters, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) {
+      set_error("%s: cudaMemsetAsync: %s", who, cudaGetErrorString(e));
+      cudaGetLastError();
+      return RA_ECUDA;
+    }
+  }
+  q_delta_kernel<<<p.grid, THREADS, SMEM_ALLOC, static_cast<cudaStream_t>(stream)>>>(p);
+  return launch_status(who);
+}
+
+}  // namespace qd
+}  // namespace ra
+
+extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
+                                      float eps, float* d_out, void* workspace, size_t workspace_bytes,
+                                      void* stream) {
+  using namespace ra;
+  clear_error();
+  const char* who = "refadapt_q_delta";
+  const ra_status v = qd::validate(who, q_cur, q_prev, B, H, d, eps, d_out);
+  if (v != RA_OK) return v;
+  if (!workspace || reinterpret_cast<uintptr_t>(workspace) % 16 != 0 ||
+      workspace_bytes < refadapt_q_delta_workspace_size(B, H)) {
+    set_error("%s: workspace must be non-NULL, 16-byte aligned and >= %zu bytes", who,
+              refadapt_q_delta_workspace_size(B, H));
+    return RA_EINVAL;
+  }
+  return qd::launch(who, q_cur, q_prev, B, H, d, eps, d_out, workspace, false, stream);
 }
 
 // ---------------------------------------------------------------------------
 // No-allocation variant: the workspace is a file-scope static device array.
 // Host code must not hand the array's name to a kernel (it is a host-side
-// stand-in); the device address comes from cudaGetSymbolAddress, looked up
-// once per device with that device current.
+// stand-in); the device address comes from cudaGetSymbolAddress with the
+// device current, looked up once per CUDA context (a context torn down by
+// cudaDeviceReset and created again gets the address looked up anew).
 namespace ra {
 namespace qd {
 
@@ -660,28 +694,37 @@ constexpr size_t kNoAllocBytes = kNoAllocCounterBytes + size_t(kNoAllocMaxBH) * 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 
 namespace {
+struct NoAllocSlot {
+  uint64_t ctx_id;  // context the address belongs to; 0 = none looked up yet
+  void* ptr;
+};
 std::mutex g_noalloc_mu;
-void* g_noalloc_ptr[64] = {nullptr};
+NoAllocSlot g_noalloc[64] = {};
 }  // namespace
 
-// Device address of g_noalloc_scratch on the current device (nullptr + error on failure).
+// Device address of g_noalloc_scratch in the current context (nullptr + error on failure).
 void* noalloc_scratch() {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
     set_error("refadapt_q_delta_noalloc: no usable current device");
     return nullptr;
   }
+  const uint64_t ctx = current_context_id();  // 0: unknown, look the address up every call
   std::lock_guard<std::mutex> lk(g_noalloc_mu);
-  if (g_noalloc_ptr[dev] == nullptr) {
+  NoAllocSlot& slot = g_noalloc[dev];
+  if (ctx == 0 || slot.ctx_id != ctx || slot.ptr == nullptr) {
     void* ptr = nullptr;
     const cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
     if (e != cudaSuccess || ptr == nullptr) {
+      cudaGetLastError();
       set_error("refadapt_q_delta_noalloc: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
       return nullptr;
     }
-    g_noalloc_ptr[dev] = ptr;
+    slot.ctx_id = ctx;
+    slot.ptr = ptr;
   }
-  return g_noalloc_ptr[dev];
+  return slot.ptr;
 }
 
 }  // namespace qd
@@ -691,20 +734,18 @@ extern "C" ra_status refadapt_q_delta_noalloc(const ra_seg* q_cur, const ra_seg*
                                               int32_t d, float eps, float* d_out, void* stream) {
   using namespace ra;
   clear_error();
-  if (B < 1 || H < 1 || int64_t(B) * H > qd::kNoAllocMaxBH) {
-    set_error("refadapt_q_delta_noalloc: B * H = %lld outside [1, %d], the size of the static scratch; "
-              "use refadapt_q_delta with a workspace",
-              (long long)B * H, qd::kNoAllocMaxBH);
+  const char* who = "refadapt_q_delta_noalloc";
+  const ra_status v = qd::validate(who, q_cur, q_prev, B, H, d, eps, d_out);
+  if (v != RA_OK) return v;
+  if (int64_t(B) * H > qd::kNoAllocMaxBH) {
+    set_error("%s: B * H = %lld exceeds %d, the size of the static scratch; use refadapt_q_delta with a "
+              "workspace",
+              who, (long long)B * H, qd::kNoAllocMaxBH);
     return RA_EINVAL;
   }
   void* scratch = qd::noalloc_scratch();
   if (scratch == nullptr) return RA_ECUDA;
-  // The ticket counters must start at zero; the array keeps the last call's contents.
-  const size_t counters = ((size_t(B) * H * sizeof(uint32_t)) + 255) / 256 * 256;
-  const cudaError_t e = cudaMemsetAsync(scratch, 0, counters, static_cast<cudaStream_t>(stream));
-  if (e != cudaSuccess) {
-    set_error("refadapt_q_delta_noalloc: cudaMemsetAsync: %s", cudaGetErrorString(e));
-    return RA_ECUDA;
-  }
-  return refadapt_q_delta(q_cur, q_prev, B, H, d, eps, d_out, scratch, qd::kNoAllocBytes, stream);
+  // The array keeps the last call's contents: the multi-block path clears its
+  // ticket counters before its kernel (the cluster path does not touch it).
+  return qd::launch(who, q_cur, q_prev, B, H, d, eps, d_out, scratch, true, stream);
 }

@@ -66,6 +66,35 @@ int main(void) {
     assert got == want
 
 
+def test_constants_match_c(tmp_path):
+    """Every constant the binding copies from the header has the header's value."""
+    from paper_2609_32415_gb300 import _lib
+    src = tmp_path / "consts.c"
+    src.write_text(r'''
+#include <stdio.h>
+#include "refadapt.h"
+int main(void) {
+  printf("%d %d\n", (int)RA_Q_DELTA_NOALLOC_MAX_BH, (int)RA_MASS_TILE_ROWS);
+  printf("%d %d %d %d %d\n", (int)RA_OK, (int)RA_EINVAL, (int)RA_EUNSUPPORTED, (int)RA_ECUDA, (int)RA_ETIMEOUT);
+  printf("%d %d %d %d\n", (int)RA_MODE_REUSE, (int)RA_MODE_BOUNDARY, (int)RA_MODE_COMPUTE, (int)RA_MODE_FULL);
+  printf("%d %d %d %d %d %d\n", (int)RA_TEXT, (int)RA_REF, (int)RA_TGT, (int)RA_CUE_PRODUCT, (int)RA_CUE_CHANGE,
+         (int)RA_CUE_EXPOSURE);
+  printf("%d %d %d %d\n", (int)RA_EPI_STORE, (int)RA_EPI_GELU, (int)RA_EPI_RESID, (int)RA_EPI_QKV);
+  return 0;
+}
+''')
+    exe = tmp_path / "consts"
+    subprocess.run(["gcc", "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe)],
+                   check=True)
+    got = [int(x) for x in subprocess.run([str(exe)], capture_output=True, text=True, check=True).stdout.split()]
+    want = [_lib.RA_Q_DELTA_NOALLOC_MAX_BH, _lib.RA_MASS_TILE_ROWS,
+            _lib.RA_OK, _lib.RA_EINVAL, _lib.RA_EUNSUPPORTED, _lib.RA_ECUDA, _lib.RA_ETIMEOUT,
+            _lib.RA_MODE_REUSE, _lib.RA_MODE_BOUNDARY, _lib.RA_MODE_COMPUTE, _lib.RA_MODE_FULL,
+            _lib.RA_TEXT, _lib.RA_REF, _lib.RA_TGT, _lib.RA_CUE_PRODUCT, _lib.RA_CUE_CHANGE, _lib.RA_CUE_EXPOSURE,
+            _lib.RA_EPI_STORE, _lib.RA_EPI_GELU, _lib.RA_EPI_RESID, _lib.RA_EPI_QKV]
+    assert got == want
+
+
 def test_dit_struct_layouts_match_c(tmp_path):
     """The GEMM and modulated-LayerNorm argument structs agree between the C
     header and the ctypes binding."""

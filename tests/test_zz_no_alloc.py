@@ -2,7 +2,9 @@
 device memory (for example a plugin whose host framework owns the device
 memory pool, or a latency-critical loop that must not pay cudaMalloc's implicit
 synchronisation). Its scratch is a static array inside the library; the result
-must match refadapt_q_delta with a caller-owned workspace, call after call.
+must equal refadapt_q_delta with a caller-owned workspace bit for bit, call
+after call (both run the same fixed-order reduction on the same inputs), and
+Eq. 1 as the oracle computes it within the Q-change tolerance.
 
 This file sorts last so that a run stopping at the first failure has already
 run every other test; it also passes on its own in a fresh process."""
@@ -10,7 +12,8 @@ import numpy as np
 import pytest
 import torch
 
-from _helpers import D_REL
+import oracle
+from _helpers import D_REL, f64
 
 pytestmark = pytest.mark.gpu
 
@@ -21,6 +24,17 @@ def _pair(g, B, H, n, d, drift):
     return cur.cuda(), prev.cuda()
 
 
+def _both(cur, prev, ws):
+    from paper_2609_32415_gb300 import api
+    B, H = cur.shape[:2]
+    want = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
+    got = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
+    api.refadapt_q_delta(cur, prev, want, ws, 1e-6)
+    api.refadapt_q_delta_noalloc(cur, prev, got, 1e-6)
+    torch.cuda.synchronize()
+    return got, want
+
+
 def test_noalloc_matches_workspace_entry_point_twice(cuda_ok):
     from paper_2609_32415_gb300 import api
     B, H, d = 2, 24, 128
@@ -28,14 +42,11 @@ def test_noalloc_matches_workspace_entry_point_twice(cuda_ok):
     ws = api.q_delta_workspace(B, H)
     for call, (n, drift) in enumerate([(1000, 0.3), (4096, 0.05)]):
         cur, prev = _pair(g, B, H, n, d, drift)
-        want = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
-        got = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
-        api.refadapt_q_delta(cur, prev, want, ws, 1e-6)
-        api.refadapt_q_delta_noalloc(cur, prev, got, 1e-6)
-        torch.cuda.synchronize()
-        w, o = want.double().cpu().numpy(), got.double().cpu().numpy()
-        assert np.all(np.isfinite(o)), call
-        assert (np.abs(o - w) / np.abs(w)).max() <= D_REL, call
+        got, want = _both(cur, prev, ws)
+        assert torch.isfinite(got).all(), call
+        assert torch.equal(got, want), call
+        ref = oracle.q_change(f64(cur), f64(prev), 1e-6)
+        assert (np.abs(got.double().cpu().numpy() - ref) / np.abs(ref)).max() <= D_REL, call
 
 
 def test_noalloc_rejects_sizes_beyond_its_scratch(cuda_ok):
@@ -50,18 +61,16 @@ def test_noalloc_rejects_sizes_beyond_its_scratch(cuda_ok):
 
 
 def test_noalloc_long_slab_uses_the_static_scratch(cuda_ok):
-    """A slab too long for one cluster of CTAs goes through the path that needs
-    scratch (per-slab tickets and partial sums): the static array serves it."""
+    """Slabs too long for one cluster of CTAs go through the path that needs
+    scratch (per-slab tickets and partial sums): the static array serves it,
+    on two calls in a row with different slab counts and lengths."""
     from paper_2609_32415_gb300 import api
-    B, H, d = 1, 2, 128
+    d = 128
     g = torch.Generator().manual_seed(22)
-    ws = api.q_delta_workspace(B, H)
-    for n in (100000, 120000):
+    for B, H, n in ((1, 2, 100000), (2, 3, 120000)):
         cur, prev = _pair(g, B, H, n, d, 0.2)
-        want = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
-        got = torch.full((B, H), float("nan"), dtype=torch.float32, device="cuda")
-        api.refadapt_q_delta(cur, prev, want, ws, 1e-6)
-        api.refadapt_q_delta_noalloc(cur, prev, got, 1e-6)
-        torch.cuda.synchronize()
-        w, o = want.double().cpu().numpy(), got.double().cpu().numpy()
-        assert (np.abs(o - w) / np.abs(w)).max() <= D_REL, n
+        got, want = _both(cur, prev, api.q_delta_workspace(B, H))
+        assert torch.isfinite(got).all(), n
+        assert torch.equal(got, want), n
+        ref = oracle.q_change(f64(cur), f64(prev), 1e-6)
+        assert (np.abs(got.double().cpu().numpy() - ref) / np.abs(ref)).max() <= D_REL, n
