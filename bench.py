@@ -3,20 +3,26 @@
 
 One step = Algorithm 1 over every block of the workload's block stack: target
 Q change, gate, reference-cache materialisation and joint attention with the
-reference mass (all through the C ABI). Default workload: the multi-reference
-image-edit shape (60 blocks, H=24, d=128, text 256 + 2x4096 reference + 4096
-target tokens, 8 denoising steps), synthetic seeded bf16 inputs pre-generated
-in HBM for every step (each block's inputs, 231 MB, exceed L2).
+reference mass (all through the C ABI). Default workload: the video shape
+(40 blocks, H=24, d=128, text 512 + 16,380 reference + 16,380 target tokens,
+4 denoising steps, per-head target-to-reference logit bias), the largest
+configuration; synthetic seeded bf16 inputs pre-generated in HBM for every
+step of the trajectory (each block's inputs, 613 MB, exceed L2).
 
-Timed steps cycle through the 8-step trajectory (step 0 is a full refresh),
-so --steps 8 times every step of one trajectory once. The same steps are also
-timed with an always-refresh gate (delta_max = 1) for the speedup.
+Timed steps cycle through the trajectory (step 0 is a full refresh), so
+--steps 4 times every step of the video trajectory once. The same steps are
+also timed with an always-refresh gate (delta_max = 1) for the speedup, and
+with every launch on one stream in Algorithm 1's block order (the schedule a
+model whose block b query depends on block b - 1 allows).
 
-Prints one JSON line (rank 0). Its "dit_stack" object times the same
-algorithm over a stack of random-weight DiT blocks around the attention (QKV,
-output projection, MLP, LayerNorms; --dit prints that measurement as its own
-line with the CPU oracle beside it; --no-dit skips it). --impl reference times
-the CPU oracle instead (a bounded sample per step, extrapolated).
+Prints one JSON line (rank 0). Its "workloads" object carries the image-edit
+(60 blocks, 256 + 2x4096 + 4096 tokens, 8 steps) and heavy-reference (60
+blocks, 256 + 4x4096 + 4096 tokens, 8 steps) workloads timed the same way in
+the same run; its "dit_stack" object times the same algorithm over a stack of
+random-weight DiT blocks around the attention on the image-edit row partition
+(QKV, output projection, MLP, LayerNorms; --dit prints that measurement as its
+own line with the CPU oracle beside it; --no-dit skips it). --impl reference
+times the CPU oracle instead (a bounded sample per step, extrapolated).
 """
 import argparse
 import hashlib
@@ -48,11 +54,15 @@ def parse_args():
     ap.add_argument("--steps", type=int, default=8)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--config", default="c2", choices=sorted(WORKLOAD_NAMES))
+    ap.add_argument("--config", default="c3", choices=sorted(WORKLOAD_NAMES))
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-refresh-baseline", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-serial", action="store_true",
+                    help="skip the one-stream (no overlap) timing of the same steps")
+    ap.add_argument("--no-nested", action="store_true",
+                    help="skip the image-edit and heavy-reference workloads the video run nests in its line")
     ap.add_argument("--cpu-budget-s", type=float, default=12.0)
     ap.add_argument("--sweep", action="store_true",
                     help="time the sweep workload grid (tokens x reference fraction x reuse fraction); "
@@ -268,15 +278,19 @@ def union_length(intervals):
 
 
 def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False, clocks=None,
-                    barrier=None, cue="product", theta=None, diagnostics=False, diag_row_stride=8):
-    """Run warmup + timed steps (cycling the trajectory); returns timing dict."""
+                    barrier=None, cue="product", theta=None, diagnostics=False, diag_row_stride=8, overlap=True):
+    """Run warmup + timed steps (cycling the trajectory); returns timing dict.
+    overlap=False keeps every launch of a step on one stream in Algorithm 1's
+    block order (each block's Q change, gate, cache update, then attention):
+    the schedule a model whose block b query comes from block b - 1 allows."""
     import torch
     from paper_2609_32415_gb300 import Executor, roles_from_joint
     dm = wl.delta_max if delta_max is None else delta_max
     th = wl.theta if theta is None else theta
     ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, th, dm, wl.eps,
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
-                  log_steps=wl.n_steps, cue=cue, diagnostics=diagnostics, diag_row_stride=diag_row_stride)
+                  log_steps=wl.n_steps, cue=cue, diagnostics=diagnostics, diag_row_stride=diag_row_stride,
+                  overlap=overlap)
     views = [[roles_from_joint(inputs[t][b], wl.offsets(), wl.n) for b in range(wl.n_blocks)]
              for t in range(wl.n_steps)]
     T = wl.n_steps
@@ -371,18 +385,31 @@ def time_graphs(wl, inputs, warmup, steps):
 
 
 def time_e2e(wl, inputs, warmup, steps):
-    """Same steps through the public API with host-resident inputs. Per step:
-    the step's gates run first on every block's target Q (copied during the
-    previous step, behind that block's data) (Executor.gate_block: a gate
-    reads only that block's target queries, its
+    """Same steps through the public API with host-resident inputs and results.
+
+    Host side: one page-locked buffer per (step, block) with that block's
+    inputs, written by the CPU (a staging copy from the device-generated
+    trajectory, then a host memcpy), and one page-locked output buffer per
+    block. Per step: the step's gates run first on every block's target Q
+    (copied during the previous step, behind that block's data)
+    (Executor.gate_block: a gate reads only that block's target queries, its
     previous-step mass partials and the controller state of the blocks before
-    it); one device->host read of the step's modes (and gbar) follows, and
-    then, per block, the text Q/K/V and target K/V are copied, plus the
-    reference Q/K/V only when a sample materialises (a reusing block reads its
-    reference K/V from the cache), on a copy stream, triple-buffered and
-    overlapped with the attentions (Executor.attend_block), up to two blocks
-    ahead; consecutive attentions alternate between two high-priority
-    streams."""
+    it); one device->host read of the step's modes (and gbar) follows; then,
+    per block, the text Q/K/V and target K/V are copied, plus the reference
+    Q/K/V only when a sample materialises (a reusing block reads its reference
+    K/V from the cache), on a copy stream, triple-buffered and overlapped with
+    the attentions (Executor.attend_block), up to two blocks ahead;
+    consecutive attentions alternate between two high-priority streams; every
+    executed row of the block's attention output (text and target rows, and
+    reference rows where a sample materialised) goes back to the host on a
+    second copy stream as soon as the attention ends. A step ends when its
+    last output is on the host.
+
+    Two measurements over the same buffers: the first trajectory right after
+    the host buffers were written (no untimed pass over them: what a caller's
+    first trajectory sees, with the device's translations of freshly pinned
+    host memory still cold), then, after `warmup` more steps, `steps` timed
+    steps (steady state)."""
     import torch
     from paper_2609_32415_gb300 import Executor
     T, nb = wl.n_steps, wl.n_blocks
@@ -393,14 +420,6 @@ def time_e2e(wl, inputs, warmup, steps):
     shape = {r: (wl.B, wl.H, wl.n[r], wl.d) for r in ROLES}
     size = {k: sum(math.prod(shape[r]) for _, r in v) for k, v in parts.items()}
     per_block = size["tq"] + size["base"] + size["ref"]
-    # Page-locked host copy of the trajectory (cudaHostAlloc through torch's
-    # pinned allocator), one buffer per (step, block). On the hosts used here
-    # the first ~16 GB of pinned memory a process allocates copies at ~25 GB/s
-    # when its device-side translations are cold (the rest at the link's ~210
-    # GB/s; a warm copy of the same range is fast, so a rate probe cannot see
-    # it): that range is allocated first and left unused.
-    parked = torch.empty(8 << 30, dtype=torch.bfloat16, pin_memory=True)
-    bufs = [[torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True) for _ in range(nb)] for _ in range(T)]
 
     def views(flat, start, kind):
         out, o = {}, start
@@ -409,46 +428,61 @@ def time_e2e(wl, inputs, warmup, steps):
             o += math.prod(shape[r])
         return out
 
-    host = []
     o_base, o_ref = size["tq"], size["tq"] + size["base"]
+    # Page-locked host trajectory (cudaHostAlloc through torch's pinned
+    # allocator), written by the CPU: each block's bytes go device -> a
+    # staging buffer, then a host memcpy into the block's own buffer.
+    stage = torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True)
+    stage_v = {"tq": views(stage, 0, "tq"), "base": views(stage, o_base, "base"), "ref": views(stage, o_ref, "ref")}
+    bufs, host = [], []
     for t in range(T):
-        row = []
+        brow, hrow = [], []
         for b in range(nb):
             X = inputs[t][b]
-            v = {"tq": views(bufs[t][b], 0, "tq"), "base": views(bufs[t][b], o_base, "base"),
-                 "ref": views(bufs[t][b], o_ref, "ref")}
-            for kind in v:
-                for (z, r), h in v[kind].items():
+            for kind in stage_v:
+                for (z, r), h in stage_v[kind].items():
                     h.copy_(X[z, :, :, off[r]:off[r] + wl.n[r], :])
-            row.append({k: bufs[t][b][o:o + size[k]] for k, o in (("tq", 0), ("base", o_base), ("ref", o_ref))})
-        host.append(row)
+            buf = torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True)
+            buf.copy_(stage)
+            brow.append(buf)
+            hrow.append({k: buf[o:o + size[k]] for k, o in (("tq", 0), ("base", o_base), ("ref", o_ref))})
+        bufs.append(brow)
+        host.append(hrow)
+    del stage, stage_v
+    # Page-locked host outputs, one set per block (each step overwrites them).
+    hout = [{r: torch.empty(shape[r], dtype=torch.bfloat16, pin_memory=True) for r in ROLES} for _ in range(nb)]
     torch.cuda.synchronize()
     dev = torch.device("cuda")
     # Device staging: each block's target Q for the current and the previous
-    # step (read as q_{t-1}), and NSLOT slots for the rest of a block.
+    # step (read as q_{t-1}), NSLOT slots for the rest of a block and NOUT
+    # output slots.
     tq = [[torch.empty(size["tq"], dtype=torch.bfloat16, device=dev) for _ in range(nb)] for _ in range(2)]
     NSLOT = 3  # the copy stream may run two blocks ahead of the attentions
     slots = [torch.empty(size["base"] + size["ref"], dtype=torch.bfloat16, device=dev) for _ in range(NSLOT)]
     slot_v = [{**views(x, 0, "base"), **views(x, size["base"], "ref")} for x in slots]
+    NOUT = 3
+    osl = [{r: torch.empty(shape[r], dtype=torch.bfloat16, device=dev) for r in ROLES} for _ in range(NOUT)]
     ex = Executor(nb, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max, wl.eps,
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T)
     comp = torch.cuda.current_stream()
     copy = torch.cuda.Stream()
+    back = torch.cuda.Stream()  # device -> host results
     # consecutive blocks' attentions on two high-priority streams (as in
     # Executor.step): block b + 1 may start in block b's last wave
     lo_pri, hi_pri = torch.cuda.Stream.priority_range()
     attn_streams = [torch.cuda.Stream(priority=hi_pri) for _ in range(2)]
     gates_done = torch.cuda.Event()
     attn_join = [torch.cuda.Event() for _ in range(2)]
+    back_join = torch.cuda.Event()
     slot_free = [torch.cuda.Event() for _ in range(NSLOT)]
+    out_free = [torch.cuda.Event() for _ in range(NOUT)]
     tq_free = [torch.cuda.Event() for _ in range(2)]
-    for e in slot_free + tq_free:
+    for e in slot_free + out_free + tq_free:
         e.record(comp)
     modes_host = torch.empty((nb, wl.B), dtype=torch.int32, pin_memory=True)
     gbar_host = torch.empty((nb, wl.B), dtype=torch.float32, pin_memory=True)
-    d2h = modes_host.numel() * 4 + gbar_host.numel() * 4
     decided = torch.cuda.Event()
-    h2d = [0]
+    h2d, d2h = [0], [0]
     PREFETCH = NSLOT  # blocks whose text and target K/V are copied before the step's modes are read
 
     def copy_base(t, b, s):
@@ -482,6 +516,7 @@ def time_e2e(wl, inputs, warmup, steps):
         tq_free[1 - p].record(comp)  # the gates of this step have read the previous step's queries
         modes_host.copy_(ex.modes[li], non_blocking=True)
         gbar_host.copy_(ex.gbar[li], non_blocking=True)
+        d2h[0] += modes_host.numel() * 4 + gbar_host.numel() * 4
         decided.record(comp)
         first = counter[0]
         for b in range(min(PREFETCH, nb)):
@@ -494,6 +529,7 @@ def time_e2e(wl, inputs, warmup, steps):
         copy.wait_event(tq_free[1 - p])  # the next step's queries go where the previous step's were
         for b in range(nb):
             s = counter[0] % NSLOT
+            o = counter[0] % NOUT
             counter[0] += 1
             if b >= PREFETCH:
                 copy_base(t, b, s)
@@ -506,48 +542,65 @@ def time_e2e(wl, inputs, warmup, steps):
             tq_ready[1 - p] = copy_tq(t_next, 1 - p, [b])  # the next step's target Q of this block, behind its data
             st = attn_streams[b % 2]
             st.wait_event(ready)
+            st.wait_event(out_free[o])
             sv = slot_v[s]
             x = {"text": (sv[(0, "text")], sv[(1, "text")], sv[(2, "text")]),
                  "ref": (sv[(0, "ref")], sv[(1, "ref")], sv[(2, "ref")]),
                  "tgt": (tq[p][b].view(shape["tgt"]), sv[(1, "tgt")], sv[(2, "tgt")])}
             with torch.cuda.stream(st):
-                ex.attend_block(t, b, x, ex.scratch_outputs(b % 2), log_index=li)
+                ex.attend_block(t, b, x, osl[o], log_index=li)
                 slot_free[s].record(st)
+                done = torch.cuda.Event()
+                done.record(st)
+            back.wait_event(done)
+            with torch.cuda.stream(back):
+                for r in (("text", "ref", "tgt") if need_ref[b] else ("text", "tgt")):
+                    hout[b][r].copy_(osl[o][r], non_blocking=True)
+                    d2h[0] += osl[o][r].numel() * 2
+                out_free[o].record(back)
         for st, j in zip(attn_streams, attn_join):  # the next step's gates read this step's mass partials
             j.record(st)
             comp.wait_event(j)
+        back_join.record(back)  # the step ends when its last result is on the host
+        comp.wait_event(back_join)
 
-    # One untimed copy of every host buffer first: the first transfer from a
-    # freshly registered range also sets up its device-side translations.
-    for t in range(T):
-        for b in range(nb):
-            slots[0][:per_block - size["tq"]].copy_(bufs[t][b][size["tq"]:], non_blocking=True)
-            tq[0][0].copy_(host[t][b]["tq"], non_blocking=True)
-    torch.cuda.synchronize()
     counter = [0, 0]  # blocks, steps
-    seq = [i % T for i in range(warmup + steps + 1)]
+    seq = [i % T for i in range(T + warmup + steps + 1)]
+
+    def timed(k0, k):
+        h2d[0] = d2h[0] = 0
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(k + 1)]
+        ev[0].record()
+        for i in range(k):
+            one_step(seq[k0 + i], counter, seq[k0 + i + 1])
+            ev[i + 1].record()
+        torch.cuda.synchronize()
+        return (ev[0].elapsed_time(ev[-1]) / k, [round(ev[i].elapsed_time(ev[i + 1]), 3) for i in range(k)],
+                int(h2d[0] // k), int(d2h[0] // k))
+
+    torch.cuda.synchronize()
+    first_ms, first_steps, first_h2d, first_d2h = timed(0, T)
     for i in range(warmup):
-        one_step(seq[i], counter, seq[i + 1])
+        one_step(seq[T + i], counter, seq[T + i + 1])
     torch.cuda.synchronize()
-    h2d[0] = 0
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(steps + 1)]
-    ev[0].record()
-    for k in range(steps):
-        one_step(seq[warmup + k], counter, seq[warmup + k + 1])
-        ev[k + 1].record()
-    torch.cuda.synchronize()
+    ms, per_step, h2d_b, d2h_b = timed(T + warmup, steps)
     ex.check()
-    ms = ev[0].elapsed_time(ev[-1])
-    per_step = [round(ev[k].elapsed_time(ev[k + 1]), 3) for k in range(steps)]
-    del host, slots, slot_v, tq, ex, bufs, parked
-    return {"value": ms / steps, "unit": "ms/step", "per_step_ms": per_step, "h2d_bytes_per_step": int(h2d[0] // steps),
-            "d2h_bytes_per_step": int(d2h),
-            "host_buffers": "pinned (cudaHostAlloc), one per (step, block), allocated after a 16 GB pinned "
-                            "range left unused",
-            "pipeline": "per step: the step's gates first (every block's target Q copied during the previous "
-                        "step), one read of the modes, then per block text Q/K/V + target K/V and reference "
-                        "Q/K/V only where a sample materialises, plus the next step's target Q; h2d bytes are "
-                        "the mean over the timed steps"}
+    del host, slots, slot_v, osl, tq, ex, bufs, hout
+    pipeline = ("per step: the step's gates first (every block's target Q copied during the previous step), one "
+                "read of the modes, then per block text Q/K/V + target K/V and reference Q/K/V only where a "
+                "sample materialises, plus the next step's target Q; every executed output row (text and target, "
+                "reference where a sample materialised) back to the host behind each attention; bytes are the "
+                "mean over the timed steps")
+    return {"value": ms, "unit": "ms/step", "per_step_ms": per_step, "h2d_bytes_per_step": h2d_b,
+            "d2h_bytes_per_step": d2h_b,
+            "host_buffers": "pinned (cudaHostAlloc), one per (step, block) and one output set per block, written "
+                            "by the CPU; timed after the first trajectory over them and %d warm-up steps" % warmup,
+            "pipeline": pipeline,
+            "first_use": {"value": first_ms, "unit": "ms/step", "per_step_ms": first_steps,
+                          "h2d_bytes_per_step": first_h2d, "d2h_bytes_per_step": first_d2h,
+                          "steps": T,
+                          "host_buffers": "the same buffers, timed from their first use: no untimed pass over "
+                                          "them, no pinned range set aside"}}
 
 
 def _q_delta_launch_ms(pairs, B, H, eps, reps):
@@ -661,6 +714,72 @@ def cpu_oracle_sample(wl, X, budget_s):
             "threads": nth, "sample_s": elapsed}
 
 
+def make_wl(name, rank=0, blocks=0):
+    """The named workload with this rank's seed (replicas draw their own
+    trajectories), optionally cut to its first `blocks` blocks."""
+    from paper_2609_32415_gb300 import synth
+    wl = synth.make_workload(name, seed=rank) if name in ("c3", "c4") else synth.make_workload(name)
+    if name not in ("c3", "c4"):
+        wl.seed = rank
+    if blocks > 0:
+        wl.n_blocks = min(wl.n_blocks, blocks)
+        wl.ref_drift = wl.ref_drift[:wl.n_blocks]
+        wl.tgt_drift = wl.tgt_drift[:wl.n_blocks]
+    return wl
+
+
+def config_dict(wl, args, ws):
+    """The line's `config` (both arms print the same one)."""
+    return {"workload": WORKLOAD_NAMES[wl.name] + (" (first %d blocks)" % wl.n_blocks if args.blocks > 0 else ""),
+            "name": wl.name, "B": wl.B, "H": wl.H, "d": wl.d,
+            "tokens": {"text": wl.n_text, "ref": wl.n_ref, "tgt": wl.n_tgt},
+            "blocks": wl.n_blocks, "trajectory_steps": wl.n_steps, "theta": round(wl.theta, 6),
+            "delta_max": wl.delta_max,
+            "l2": "inputs larger than L2 (%.0f MB per block)" % (3 * wl.B * wl.H * wl.N * wl.d * 2 / 1e6),
+            "resident_steps": wl.n_steps,
+            "parallelism": "replicas" if ws > 1 else "single GPU"}
+
+
+def q_delta_summary(qd, peaks):
+    return {"bound": "hbm", "kernel": "q_delta_cluster_kernel", "achieved": round(qd["gbs"], 1),
+            "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(qd["gbs"] / peaks["hbm_gbs"], 4),
+            "bytes_per_launch": qd["bytes"], "launch_ms": round(qd["ms"], 5),
+            "same_bytes_torch_sum_gbs": round(qd["lib_read_gbs"], 1),
+            "peak_kind": "%s HBM copy" % peaks["source"]}
+
+
+def run_nested(name, args, peaks):
+    """Another workload timed the same way inside the same run (attention-only
+    steps, gated and always-refresh, and the Q change): one object of the
+    line."""
+    import torch
+    wl = make_wl(name)
+    inputs = make_inputs(wl, "cuda")
+    torch.cuda.synchronize()
+    clocks = Clocks(0)
+    main = time_trajectory(wl, inputs, args.warmup, args.steps, attn_timing=True, clocks=clocks)
+    refresh = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1)
+    qd = time_q_delta(wl, inputs)
+    del inputs
+    torch.cuda.empty_cache()
+    ms = main["total_ms"] / args.steps
+    tf = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
+    sched = expected_schedule(wl)
+    return {"workload": WORKLOAD_NAMES[name], "name": name, "blocks": wl.n_blocks,
+            "trajectory_steps": wl.n_steps, "theta": round(wl.theta, 6), "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms, 3),
+            "per_step_ms": [round(x, 3) for x in main["per_step_ms"]],
+            "modes_per_step": {str(t): [int(x) for x in main["modes"][t, :, 0]] for t in sorted(set(main["steps_t"]))},
+            "schedule_matches_expected": all([int(x) for x in main["modes"][t, :, 0]] == sched[t]
+                                             for t in set(main["steps_t"])),
+            "attn_tflops": round(tf, 1), "attn_frac_of_bf16_peak": round(tf / peaks["bf16_sustained"], 4),
+            "attn_launch_ms": round(main["attn_ms"] / main["attn_launches"], 4),
+            "always_refresh_ms_per_step": round(refresh["total_ms"] / args.steps, 3),
+            "speedup_vs_always_refresh": round(refresh["total_ms"] / main["total_ms"], 3),
+            "q_delta_roofline": q_delta_summary(qd, peaks),
+            "clocks": main["clocks"]}
+
+
 def main_ours(args):
     import torch
     import torch.distributed as dist
@@ -674,14 +793,7 @@ def main_ours(args):
     else:
         barrier = None
     ge.build()
-    wl = synth.make_workload(args.config, seed=rank) if args.config in ("c3", "c4") else \
-        synth.make_workload(args.config)
-    if args.config not in ("c3", "c4"):
-        wl.seed = rank
-    if args.blocks > 0:
-        wl.n_blocks = min(wl.n_blocks, args.blocks)
-        wl.ref_drift = wl.ref_drift[:wl.n_blocks]
-        wl.tgt_drift = wl.tgt_drift[:wl.n_blocks]
+    wl = make_wl(args.config, rank, args.blocks)
     peaks = load_peaks()
     inputs = make_inputs(wl, "cuda")
     torch.cuda.synchronize()
@@ -693,8 +805,11 @@ def main_ours(args):
     refresh = None
     if not args.no_refresh_baseline:
         refresh = time_trajectory(wl, inputs, args.warmup, args.steps, delta_max=1, barrier=barrier)
+    serial = None
+    if not args.no_serial:
+        serial = time_trajectory(wl, inputs, args.warmup, args.steps, overlap=False, barrier=barrier)
     qd = time_q_delta(wl, inputs)
-    qd_long = time_q_delta_long(H=wl.H, d=wl.d, eps=wl.eps) if wl.d == 128 else None
+    qd_long = time_q_delta_long(H=wl.H, d=wl.d, eps=wl.eps) if (wl.d == 128 and wl.n_tgt < 16380) else None
     diag = None
     if args.diagnostics:
         diag = time_trajectory(wl, inputs, args.warmup, args.steps, diagnostics=True, diag_row_stride=8)
@@ -721,18 +836,27 @@ def main_ours(args):
                "sample": "fp64 C oracle, %d target query rows x %d heads of block 0 (step 1) against all %d keys "
                          "(%.1f s) plus Eq. 1 over the block's target Q; extrapolated per query row to the "
                          "executed rows of the timed steps" % (s["rows"], s["heads"], wl.N, s["sample_s"])}
+    del inputs
+    torch.cuda.empty_cache()
+    nested = {}
+    if rank == 0 and ws == 1 and not args.no_nested and args.config == "c3" and args.blocks == 0:
+        for name in ("c2", "c4"):
+            try:
+                nested[name] = run_nested(name, args, peaks)
+            except Exception as exc:  # report, do not guess
+                nested[name] = {"error": str(exc)[:200]}
+            torch.cuda.empty_cache()
     dit = None
     if rank == 0 and ws == 1 and not args.no_dit:
-        # The DiT-block stack around the same attention (one line of its own with
-        # --dit); its inputs and weights replace the attention trajectory in HBM.
-        del inputs
-        torch.cuda.empty_cache()
+        # The DiT-block stack around the same attention on the image-edit row
+        # partition (one line of its own with --dit); its inputs and weights
+        # replace the attention trajectory in HBM.
         try:
-            dit_wl = synth.make_workload(args.config)
+            dit_wl = synth.make_workload("c2")
             if args.blocks > 0:
                 dit_wl.n_blocks = min(dit_wl.n_blocks, args.blocks)
             d = run_dit(args, dit_wl, with_cpu=False, with_context=False)
-            dit = {k: d[k] for k in ("value", "unit", "block", "theta", "per_step_ms", "gemm_tflops",
+            dit = {k: d[k] for k in ("workload", "value", "unit", "block", "theta", "per_step_ms", "gemm_tflops",
                                      "gemm_frac_of_bf16_peak", "gemm_share_of_step", "attn_tflops",
                                      "always_refresh_ms_per_step", "speedup_vs_always_refresh", "clocks")
                    if k in d}
@@ -746,6 +870,12 @@ def main_ours(args):
     attn_tflops = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
     traffic = recorded_traffic(args.config)
     per_launch_flops = main["attn_flops"] / main["attn_launches"]
+    qsum = q_delta_summary(qd, peaks)
+    if qd_long is not None:
+        qsum["longer_read"] = {"shape": "video target query, 16,380 rows x %d heads x d %d" % (wl.H, wl.d),
+                               "bytes_per_launch": qd_long["bytes"], "launch_ms": round(qd_long["ms"], 5),
+                               "achieved": round(qd_long["gbs"], 1),
+                               "frac": round(qd_long["gbs"] / peaks["hbm_gbs"], 4)}
     line = {
         "metric": "ms per denoising step (attention TFLOP/s and %% of bf16 peak, vs always-refresh)",
         "value": round(ms_per_step, 3),
@@ -759,13 +889,7 @@ def main_ours(args):
         "vs_baseline": None,
         "dtype": "bf16",
         "data": "synthetic (seeded bf16 Q/K/V with the workload's drift recipe; no datasets or weights)",
-        "config": {"workload": WORKLOAD_NAMES[args.config] + (
-                       " (first %d blocks)" % wl.n_blocks if args.blocks > 0 else ""),
-                   "name": args.config, "B": wl.B,
-                   "blocks": wl.n_blocks, "trajectory_steps": wl.n_steps, "theta": round(wl.theta, 6),
-                   "delta_max": wl.delta_max,
-                   "l2": "inputs larger than L2 (%.0f MB per block)" % (3 * wl.B * wl.H * wl.N * wl.d * 2 / 1e6),
-                   "parallelism": "replicas" if ws > 1 else "single GPU"},
+        "config": config_dict(wl, args, ws),
         "per_step_ms": [round(x, 3) for x in main["per_step_ms"]],
         "timed_trajectory_steps": main["steps_t"],
         "modes_per_step": {str(t): [int(x) for x in main["modes"][t, :, 0]] for t in sorted(set(main["steps_t"]))},
@@ -779,21 +903,18 @@ def main_ours(args):
                      "flops_per_launch": int(per_launch_flops),
                      "launch_ms": round(main["attn_ms"] / main["attn_launches"], 4),
                      "peak_kind": "%s, sustained bf16 (kernel timed inside a long step)" % peaks["source"]},
-        "q_delta_roofline": {"bound": "hbm", "achieved": round(qd["gbs"], 1), "peak": peaks["hbm_gbs"],
-                             "unit": "GB/s", "frac": round(qd["gbs"] / peaks["hbm_gbs"], 4),
-                             "bytes_per_launch": qd["bytes"], "launch_ms": round(qd["ms"], 5),
-                             "same_bytes_torch_sum_gbs": round(qd["lib_read_gbs"], 1),
-                             "peak_kind": "%s HBM copy" % peaks["source"],
-                             "longer_read": None if qd_long is None else {
-                                 "shape": "video target query, 16,380 rows x %d heads x d %d" % (wl.H, wl.d),
-                                 "bytes_per_launch": qd_long["bytes"], "launch_ms": round(qd_long["ms"], 5),
-                                 "achieved": round(qd_long["gbs"], 1),
-                                 "frac": round(qd_long["gbs"] / peaks["hbm_gbs"], 4)}},
+        "q_delta_roofline": qsum,
         "gpu_launches": main["launches"],
         "clocks": main["clocks"],
-        "e2e": e2e,
+        "e2e": None if e2e is None else {k: v for k, v in e2e.items() if k != "first_use"},
         "cpu_baseline": cpu,
     }
+    if e2e is not None and e2e.get("first_use") is not None:
+        line["e2e_unpadded"] = e2e["first_use"]
+    if serial is not None:
+        line["ms_per_step_serial"] = round(serial["total_ms"] / args.steps, 3)
+        line["serial_schedule"] = ("one stream, Algorithm 1's block order: each block's Q change, gate, cache "
+                                   "update, then its attention (no work of block b under block b - 1's attention)")
     if diag is not None:
         dms = diag["total_ms"] / args.steps
         line["diagnostics_ms_per_step"] = round(dms, 3)
@@ -812,6 +933,8 @@ def main_ours(args):
     sched = expected_schedule(wl)
     line["schedule_matches_expected"] = all(
         [int(x) for x in main["modes"][t, :, 0]] == sched[t] for t in set(main["steps_t"]))
+    if nested:
+        line["workloads"] = nested
     if dit is not None:
         line["dit_stack"] = dit
     emit(line, args)
@@ -831,14 +954,16 @@ def emit(line, args):
 # ----------------------------------------------------------------------------- reference arm
 def main_reference(args):
     """The CPU oracle as it stands, on the host cores: each step a bounded sample
-    of the workload, extrapolated to one denoising step."""
+    of the workload, extrapolated to one denoising step over the schedule the
+    workload's recipe gives (the GPU arm reports whether its executed schedule
+    is that one: schedule_matches_expected)."""
     ws, rank, _ = dist_env()
     if rank != 0:
         return
     from oracle import build as oracle_build
     from paper_2609_32415_gb300 import synth
     oracle_build.build()
-    wl = synth.make_workload(args.config)
+    wl = make_wl(args.config, 0, args.blocks)
     sched = expected_schedule(wl)
     traj = synth.Trajectory(wl, device="cpu")
     X = traj.get(1, 0)
@@ -860,11 +985,12 @@ def main_reference(args):
         "value": value, "unit": "ms/step", "n_gpus": ws, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": value, "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
         "dtype": "f64", "data": "synthetic (seeded bf16 inputs widened to fp64)",
-        "config": {"workload": WORKLOAD_NAMES[args.config], "name": args.config},
+        "config": config_dict(wl, args, ws),
+        "schedule": {str(t): sched[t] for t in range(wl.n_steps)},
         "cpu_baseline": {"value": value, "unit": "ms/step", "cores": last["threads"], "kind": "oracle",
                          "sample": "per step: %d target query rows x %d heads of one block against all %d keys "
-                                   "plus Eq. 1 over the block's target Q, extrapolated to the workload's expected "
-                                   "schedule of executed rows" % (last["rows"], last["heads"], wl.N)},
+                                   "plus Eq. 1 over the block's target Q, extrapolated to the executed rows of "
+                                   "the workload's schedule" % (last["rows"], last["heads"], wl.N)},
         "e2e": {"value": value, "unit": "ms/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     emit(line, args)
@@ -1127,7 +1253,7 @@ def run_dit(args, wl, with_cpu=True, with_context=True):
     at = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
     ms = main["total_ms"] / args.steps
     line = {
-        "workload": "DiT-block stack: " + WORKLOAD_NAMES[args.config] + (
+        "workload": "DiT-block stack: " + WORKLOAD_NAMES[wl.name] + (
             " (first %d blocks)" % wl.n_blocks if args.blocks > 0 else ""),
         "block": "dual-stream MMDiT, C=%d, MLP 4C, random weights (%.1f GB)" % (
             C, sum(v.numel() * v.element_size() for w in tables[3] for st in w.values() for v in st.values()) / 1e9),
