@@ -146,8 +146,9 @@ int32_t refadapt_mass_partial_len(int32_t n_text, int32_t n_tgt);
  * "Runtime cues"):
  *   D[b][h] = ||q_cur - q_prev||_F / (||q_prev||_F + eps)
  * over the segment's n rows x d columns. Bandwidth-bound: reads both tensors
- * once through bulk copies into shared memory, fp32 per-thread sums, fp64
- * across threads and blocks in a fixed order (deterministic).
+ * once through bulk copies into shared memory; fp32 per-thread sums and
+ * butterflies, then compensated two-float sums across units, warps and
+ * blocks, all in a fixed order (deterministic; relative error of D ~1e-7).
  *
  * Each slab (one sample and head) is reduced by one thread-block cluster of
  * up to 8 CTAs through distributed shared memory, leaving the workspace

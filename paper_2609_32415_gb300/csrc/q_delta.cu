@@ -1,31 +1,42 @@
 // refadapt_q_delta: relative L2 change of the target query per (sample, head),
 // D = ||q_t - q_{t-1}||_F / (||q_{t-1}||_F + eps)   (paper Eq. 1, Sec. 4).
 //
-// HBM-bound streaming reduction, one CTA per SM. Work is cut into units of
-// 12 KB per tensor (48 rows at d = 128, 96 rows at d = 64) of one (sample,
-// head) slab; CTA c takes the contiguous unit range [c U / G, (c+1) U / G) in
-// slab-major order. A producer thread streams both tensors' units through an
-// 8-stage shared-memory ring, so each SM keeps up to 192 KB in flight without
-// register limits. When both tensors' rows are contiguous within a slab
-// (stride_n == d) a unit is one 1-D bulk copy of its bytes (the slab's last
-// unit is shorter); otherwise it is a 2-D TMA tensor load (any row strides;
-// rows past the slab end arrive as zeros and add nothing). Unit i goes to stage i % 8 and is
-// consumed by warp i % 8, so every stage has one consumer that waits its
-// phases in order: packed fp32 sums of (q_t - q_{t-1})^2 and q_{t-1}^2 per
-// lane, then an fp64 butterfly per unit. The CTA then adds its unit sums per
-// slab in unit order and stores one slot per (slab, CTA); the slab's last
-// contributor (ticket counter) adds the slots in CTA order and writes D, then
-// re-arms the counter. Every sum has a fixed order, so D is deterministic.
+// HBM-bound streaming reduction. Work is cut into units of 12 KB per tensor
+// (48 rows at d = 128, 96 rows at d = 64) of one (sample, head) slab. When
+// both tensors' rows are contiguous within a slab (stride_n == d) a unit is
+// one 1-D bulk copy of its bytes (the slab's last unit is shorter); otherwise
+// it is a 2-D TMA tensor load (any row strides; rows past the slab end arrive
+// as zeros and add nothing). A producer thread streams both tensors' units
+// through a shared-memory ring; unit i goes to stage i % S and is consumed by
+// warp i % S, so every stage has one consumer that waits its phases in order.
+//
+// Arithmetic stays off the FP64 pipe, which is narrow on this GPU (a chain
+// of dependent fp64 adds, square roots and a division cost microseconds at
+// the end of a launch): packed fp32 sums of (q_t - q_{t-1})^2 and q_{t-1}^2
+// per lane, an fp32 butterfly per unit, then compensated two-float sums
+// (TwoSum: hi + lo carries the rounding error of every addition) across
+// units, warps, CTAs and cluster ranks, and D formed in fp32 from hi + lo.
+// Every sum has a fixed order, so D is deterministic.
 //
 // Cluster path (used when the slabs fit clusters that fill the GPU): one
 // cluster of up to 8 CTAs per (sample, head) slab, each CTA streaming its
 // contiguous share of the slab's units through an 8-stage ring (one CTA per
 // SM) or a 4-stage ring (two per SM), whichever fills the SMs better; every
-// CTA stores its pair of sums into the cluster leader's shared memory
-// (distributed shared memory) and, after one cluster barrier, the leader adds
-// them in rank order and writes D. No global atomics, fences or workspace: the
-// reduction tail is one cluster barrier. The path above remains for slabs too
-// long for one cluster and for too few slabs to fill the GPU.
+// CTA stores its sums into the cluster leader's shared memory (distributed
+// shared memory) and, after one cluster barrier, the leader adds them in rank
+// order and writes D. No global atomics, fences or workspace: the reduction
+// tail is one cluster barrier. On the bulk path each CTA asks L2 for its
+// first S units before it waits for the previous kernel of the stream
+// (programmatic dependent launch): L2 is the GPU's point of coherence, so the
+// loads issued after that wait still see everything the previous kernel
+// wrote, and the first units no longer pay the full trip from HBM after it.
+//
+// Multi-block path (slabs too long for one cluster, or too few slabs to fill
+// the GPU): one CTA per SM, an 8-stage ring; CTA c takes the contiguous unit
+// range [c U / G, (c+1) U / G) in slab-major order, adds its unit sums per
+// slab in unit order into one slot per (slab, CTA) of the workspace; the
+// slab's last contributor (ticket counter) adds the slots in CTA order,
+// writes D and re-arms the counter.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -48,8 +59,8 @@ constexpr int THREADS = 32 * (CONSUMER_WARPS + 1);
 constexpr int MAX_UNITS_PER_CTA = 1024;
 constexpr int OFF_BAR = STAGES * 2 * UNIT_BYTES;
 constexpr int OFF_MISC = OFF_BAR + 2 * STAGES * 8;           // abort flag
-constexpr int OFF_SUMS = OFF_MISC + 16;                       // double2 per unit
-constexpr int SMEM_BYTES = OFF_SUMS + MAX_UNITS_PER_CTA * 16;
+constexpr int OFF_SUMS = OFF_MISC + 16;                       // float2 per unit
+constexpr int SMEM_BYTES = OFF_SUMS + MAX_UNITS_PER_CTA * 8;
 constexpr int SMEM_ALLOC = SMEM_BYTES + 1024;
 static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 
@@ -66,7 +77,7 @@ struct Params {
   int32_t grid;
   float eps;
   float* d_out;
-  double* partial;         // [B*H][MAX_SPLITS][2]
+  float4* partial;         // [B*H][MAX_SPLITS]: (hi, lo) of both sums
   uint32_t* counter;       // [B*H]
   uint64_t budget_ns;
 };
@@ -91,13 +102,48 @@ __device__ __forceinline__ void acc16(const uint4& c, const uint4& p, uint64_t& 
   }
 }
 
+// L2 prefetch of `bytes` (a multiple of 16) at a 16-byte aligned global address.
+__device__ __forceinline__ void bulk_prefetch_l2(const void* src, uint32_t bytes) {
+  asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(reinterpret_cast<uint64_t>(src)), "r"(bytes)
+               : "memory");
+}
+
+// (hi, lo) += x with the rounding error of the addition kept in lo (TwoSum,
+// six fp32 operations; the value is hi + lo).
+__device__ __forceinline__ void ff_add(float& hi, float& lo, float x) {
+  const float s = hi + x;
+  const float v = s - hi;
+  lo += (hi - (s - v)) + (x - v);
+  hi = s;
+}
+
+// Sum of one lane value over the warp (fixed butterfly: every lane ends with
+// the same value).
+__device__ __forceinline__ float warp_sum(float x) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+  return x;
+}
+
+// (hi, lo) pairs of the 32 lanes added up in a fixed tree; lane 0 ends with
+// the total (the other lanes' values are partial).
+__device__ __forceinline__ void ff_tree(float& hi, float& lo) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float xh = __shfl_down_sync(0xffffffffu, hi, o);
+    const float xl = __shfl_down_sync(0xffffffffu, lo, o);
+    ff_add(hi, lo, xh);
+    lo += xl;
+  }
+}
+
 __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_constant__ Params p) {
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + OFF_BAR);
   uint64_t* empty = full + STAGES;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + OFF_MISC);
-  double* sums = reinterpret_cast<double*>(smem + OFF_SUMS);
+  float* sums = reinterpret_cast<float*>(smem + OFF_SUMS);
   const int c = blockIdx.x;
   const int u0 = int(int64_t(c) * p.units / p.grid);
   const int u1 = int(int64_t(c + 1) * p.units / p.grid);
@@ -174,15 +220,10 @@ __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_consta
       float a0, a1, b0, b1;
       f2_unpack(sd, a0, a1);
       f2_unpack(sp, b0, b1);
-      double dd = double(a0) + double(a1), dp = double(b0) + double(b1);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        dd += __shfl_xor_sync(0xffffffffu, dd, o);
-        dp += __shfl_xor_sync(0xffffffffu, dp, o);
-      }
+      const float ud = warp_sum(a0 + a1), up = warp_sum(b0 + b1);
       if (lane == 0) {
-        sums[2 * i] = dd;
-        sums[2 * i + 1] = dp;
+        sums[2 * i] = ud;
+        sums[2 * i + 1] = up;
       }
     }
     named_bar_sync(1, 32 * CONSUMER_WARPS);
@@ -193,39 +234,40 @@ __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_consta
       int i = 0;
       while (i < nu) {
         const int slab = (u0 + i) / p.per_slab;
-        double td = 0.0, tp = 0.0;
+        float dh = 0.f, dl = 0.f, ph = 0.f, pl = 0.f;
         int j = i;
         for (; j < nu && (u0 + j) / p.per_slab == slab; ++j) {
-          td += sums[2 * j];
-          tp += sums[2 * j + 1];
+          ff_add(dh, dl, sums[2 * j]);
+          ff_add(ph, pl, sums[2 * j + 1]);
         }
         const int64_t first_u = int64_t(slab) * p.per_slab;
         const int64_t last_u = first_u + p.per_slab - 1;
         const int c_lo = owner(first_u, p.units, p.grid);
         const int count = owner(last_u, p.units, p.grid) - c_lo + 1;
-        double* slots = p.partial + int64_t(slab) * MAX_SPLITS * 2;
+        float4* slots = p.partial + int64_t(slab) * MAX_SPLITS;
         uint32_t last = 0;
         if (lane == 0) {
-          slots[2 * (c - c_lo)] = aborted ? NAN : td;
-          slots[2 * (c - c_lo) + 1] = tp;
+          __stcg(slots + (c - c_lo), make_float4(aborted ? NAN : dh, dl, ph, pl));
           __threadfence();
           last = (atomicAdd(p.counter + slab, 1u) == uint32_t(count - 1)) ? 1u : 0u;
         }
         last = __shfl_sync(0xffffffffu, last, 0);
         if (last) {
           __threadfence();
-          double sd = 0.0, sp = 0.0;
+          // lane q adds the slots q, q + 32, ... in order; then a fixed tree
+          // over the lanes' (hi, lo) pairs ends in lane 0
+          float sdh = 0.f, sdl = 0.f, sph = 0.f, spl = 0.f;
           for (int q = lane; q < count; q += 32) {
-            sd += __ldcg(slots + 2 * q);
-            sp += __ldcg(slots + 2 * q + 1);
+            const float4 v = __ldcg(slots + q);
+            ff_add(sdh, sdl, v.x);
+            sdl += v.y;
+            ff_add(sph, spl, v.z);
+            spl += v.w;
           }
-#pragma unroll
-          for (int o = 16; o > 0; o >>= 1) {
-            sd += __shfl_xor_sync(0xffffffffu, sd, o);
-            sp += __shfl_xor_sync(0xffffffffu, sp, o);
-          }
+          ff_tree(sdh, sdl);
+          ff_tree(sph, spl);
           if (lane == 0) {
-            p.d_out[slab] = float(sqrt(sd) / (sqrt(sp) + double(p.eps)));
+            p.d_out[slab] = sqrtf(sdh + sdl) / (sqrtf(sph + spl) + p.eps);
             p.counter[slab] = 0u;  // re-arm for the next call
           }
         }
@@ -237,22 +279,30 @@ __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_consta
 
 // ---------------------------------------------------------------- cluster path
 constexpr int CL_MAX_CS = 8;       // CTAs per cluster (portable limit)
-constexpr int CL_MAX_UNITS = 256;  // units per CTA
+constexpr int CL_MAX_UNITS = 256;  // units per CTA (longer slabs take the multi-block path)
 
-// Shared-memory layout of a cluster CTA with S stages (stage s belongs to
-// consumer warp s; warp S is the producer).
-template <int S>
+// Units of the cluster path: 8 KB per tensor for slabs of up to 2 MB, 12 KB
+// for longer ones. On a short read (image edit: 24 slabs of 1 MB) the smaller
+// first wave of requests and the finer split make a launch 2 % shorter; on a
+// long one (video: 24 slabs of 4.2 MB) the larger units stream 3 % faster.
+constexpr int CL_UNIT_SMALL = 8192;
+constexpr int64_t CL_SMALL_SLAB_BYTES = int64_t(2) << 20;
+
+// Shared-memory layout of a cluster CTA with S stages of UB-byte units per
+// tensor (stage s belongs to consumer warp s; warp S is the producer).
+template <int S, int UB>
 struct ClLayout {
   static constexpr int THREADS = 32 * (S + 1);
-  static constexpr int OFF_BAR = S * 2 * UNIT_BYTES;
+  static constexpr int OFF_BAR = S * 2 * UB;
   static constexpr int OFF_MISC = OFF_BAR + 2 * S * 8;          // abort flag
-  static constexpr int OFF_SUMS = OFF_MISC + 16;                 // double2 per unit
-  static constexpr int OFF_SLOTS = OFF_SUMS + CL_MAX_UNITS * 16;  // leader: double2 per rank
+  static constexpr int OFF_WSUM = OFF_MISC + 16;                 // float4 (hi, lo of both sums) per consumer warp
+  static constexpr int OFF_SLOTS = OFF_WSUM + S * 16;            // leader: float4 per rank
   static constexpr int BYTES = OFF_SLOTS + CL_MAX_CS * 16;
   static constexpr int ALLOC = BYTES + 1024;
 };
-static_assert(ClLayout<8>::ALLOC <= 232448, "shared memory budget");
-static_assert(2 * ClLayout<4>::ALLOC <= 232448, "two 4-stage CTAs per SM");
+static_assert(ClLayout<8, UNIT_BYTES>::ALLOC <= 232448, "shared memory budget");
+static_assert(2 * ClLayout<4, UNIT_BYTES>::ALLOC <= 232448, "two 4-stage CTAs per SM");
+static_assert(ClLayout<8, CL_UNIT_SMALL>::ALLOC <= 232448, "shared memory budget");
 
 struct ClusterParams {
   CUtensorMap tm_c, tm_p;
@@ -280,17 +330,18 @@ __device__ __forceinline__ void cluster_wait() {
   asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
-template <int S>
-__global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(const __grid_constant__ ClusterParams p) {
-  using L = ClLayout<S>;
+template <int S, int UB>
+__global__ void __launch_bounds__(ClLayout<S, UB>::THREADS)
+    q_delta_cluster_kernel(const __grid_constant__ ClusterParams p) {
+  using L = ClLayout<S, UB>;
   constexpr int CL_STAGES = S, CL_CONSUMERS = S;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + L::OFF_BAR);
   uint64_t* empty = full + CL_STAGES;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(smem + L::OFF_MISC);
-  double* sums = reinterpret_cast<double*>(smem + L::OFF_SUMS);
-  double* slots = reinterpret_cast<double*>(smem + L::OFF_SLOTS);
+  float4* wsum = reinterpret_cast<float4*>(smem + L::OFF_WSUM);
+  float4* slots = reinterpret_cast<float4*>(smem + L::OFF_SLOTS);
   uint32_t rank;
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(rank));
   const int h = blockIdx.y, b = blockIdx.z;
@@ -321,6 +372,17 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
     }
     __syncwarp();
     named_bar_arrive(2, L::THREADS);
+    if (p.bulk && lane < CL_STAGES && lane < nu) {
+      // Ask L2 for this CTA's first units while the previous kernel of the
+      // stream may still run. Only L2 is filled: the copies into shared
+      // memory start after griddepcontrol.wait, and L2 is coherent, so they
+      // see whatever that kernel writes meanwhile.
+      const int64_t off = int64_t(k0 + lane) * UB;
+      const int64_t rem = p.slab_bytes - off;
+      const uint32_t bytes = uint32_t(rem < UB ? rem : UB);
+      bulk_prefetch_l2(p.base_c + b * p.c_sb + h * p.c_sh + off, bytes);
+      bulk_prefetch_l2(p.base_p + b * p.p_sb + h * p.p_sh + off, bytes);
+    }
     asm volatile("griddepcontrol.wait;" ::: "memory");
     if (lane == 0) {
       // ---------------------------------------------------------- producer
@@ -334,17 +396,17 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
         if (i >= CL_STAGES && !mbar_wait(empty + s, ((i / CL_STAGES) - 1) & 1, ctl)) break;
         const int k = k0 + i;
         if (p.bulk) {
-          const int64_t off = int64_t(k) * UNIT_BYTES;
+          const int64_t off = int64_t(k) * UB;
           const int64_t rem = p.slab_bytes - off;
-          const uint32_t bytes = uint32_t(rem < UNIT_BYTES ? rem : UNIT_BYTES);
+          const uint32_t bytes = uint32_t(rem < UB ? rem : UB);
           mbar_arrive_expect_tx(full + s, 2 * bytes);
-          bulk_load(smem + s * 2 * UNIT_BYTES, p.base_c + b * p.c_sb + h * p.c_sh + off, bytes, full + s);
-          bulk_load(smem + s * 2 * UNIT_BYTES + UNIT_BYTES, p.base_p + b * p.p_sb + h * p.p_sh + off, bytes,
+          bulk_load(smem + s * 2 * UB, p.base_c + b * p.c_sb + h * p.c_sh + off, bytes, full + s);
+          bulk_load(smem + s * 2 * UB + UB, p.base_p + b * p.p_sb + h * p.p_sh + off, bytes,
                     full + s);
         } else {
-          mbar_arrive_expect_tx(full + s, 2 * UNIT_BYTES);
-          tma_load_4d(smem + s * 2 * UNIT_BYTES, &p.tm_c, full + s, 0, k * p.rows_per_unit, h, b);
-          tma_load_4d(smem + s * 2 * UNIT_BYTES + UNIT_BYTES, &p.tm_p, full + s, 0, k * p.rows_per_unit, h, b);
+          mbar_arrive_expect_tx(full + s, 2 * UB);
+          tma_load_4d(smem + s * 2 * UB, &p.tm_c, full + s, 0, k * p.rows_per_unit, h, b);
+          tma_load_4d(smem + s * 2 * UB + UB, &p.tm_p, full + s, 0, k * p.rows_per_unit, h, b);
         }
         ++issued;
       }
@@ -359,20 +421,21 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
     // ------------------------------------------------------------ consumers
     named_bar_sync(2, L::THREADS);  // the ring's barriers are initialised
     asm volatile("griddepcontrol.wait;" ::: "memory");  // orders the final store of D
+    float dh = 0.f, dl = 0.f, ph = 0.f, pl = 0.f;  // this warp's units, in order (lane 0)
     for (int i = warp; i < nu; i += CL_CONSUMERS) {
       const int s = i % CL_STAGES;
       if (!__all_sync(0xffffffffu, mbar_wait(full + s, (i / CL_STAGES) & 1, ctl))) break;
-      const uint4* vc = reinterpret_cast<const uint4*>(smem + s * 2 * UNIT_BYTES);
-      const uint4* vp = reinterpret_cast<const uint4*>(smem + s * 2 * UNIT_BYTES + UNIT_BYTES);
+      const uint4* vc = reinterpret_cast<const uint4*>(smem + s * 2 * UB);
+      const uint4* vp = reinterpret_cast<const uint4*>(smem + s * 2 * UB + UB);
       uint64_t sd = f2_pack(0.f, 0.f), sp = sd;
-      int nvec = UNIT_BYTES / 16;
+      int nvec = UB / 16;
       if (p.bulk) {
-        const int64_t rem = p.slab_bytes - int64_t(k0 + i) * UNIT_BYTES;
-        if (rem < UNIT_BYTES) nvec = int(rem / 16);
+        const int64_t rem = p.slab_bytes - int64_t(k0 + i) * UB;
+        if (rem < UB) nvec = int(rem / 16);
       }
-      if (nvec == UNIT_BYTES / 16) {
+      if (nvec == UB / 16) {
 #pragma unroll 8
-        for (int m = 0; m < UNIT_BYTES / 16 / 32; ++m) acc16(vc[lane + 32 * m], vp[lane + 32 * m], sd, sp);
+        for (int m = 0; m < UB / 16 / 32; ++m) acc16(vc[lane + 32 * m], vp[lane + 32 * m], sd, sp);
       } else {
         for (int v = lane; v < nvec; v += 32) acc16(vc[v], vp[v], sd, sp);
       }
@@ -381,17 +444,13 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
       float a0, a1, b0, b1;
       f2_unpack(sd, a0, a1);
       f2_unpack(sp, b0, b1);
-      double dd = double(a0) + double(a1), dp = double(b0) + double(b1);
-#pragma unroll
-      for (int o = 16; o > 0; o >>= 1) {
-        dd += __shfl_xor_sync(0xffffffffu, dd, o);
-        dp += __shfl_xor_sync(0xffffffffu, dp, o);
-      }
+      const float ud = warp_sum(a0 + a1), up = warp_sum(b0 + b1);
       if (lane == 0) {
-        sums[2 * i] = dd;
-        sums[2 * i + 1] = dp;
+        ff_add(dh, dl, ud);
+        ff_add(ph, pl, up);
       }
     }
+    if (lane == 0) wsum[warp] = make_float4(dh, dl, ph, pl);
     named_bar_sync(1, 32 * CL_CONSUMERS);
   }
   // Every CTA of the cluster has arrived (started), so the leader's shared
@@ -399,36 +458,63 @@ __global__ void __launch_bounds__(ClLayout<S>::THREADS) q_delta_cluster_kernel(c
   // leader's slot `rank`.
   cluster_wait();
   if (threadIdx.x == 0) {
-    double td = 0.0, tp = 0.0;
-    for (int i = 0; i < nu; ++i) {
-      td += sums[2 * i];
-      tp += sums[2 * i + 1];
+    float dh = 0.f, dl = 0.f, ph = 0.f, pl = 0.f;
+    for (int w = 0; w < CL_CONSUMERS; ++w) {
+      const float4 v = wsum[w];
+      ff_add(dh, dl, v.x);
+      dl += v.y;
+      ff_add(ph, pl, v.z);
+      pl += v.w;
     }
-    if (*abort_flag) td = NAN;
+    if (*abort_flag) dh = NAN;
     uint32_t remote;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(slots)), "r"(0));
-    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank), "d"(td) : "memory");
-    asm volatile("st.shared::cluster.f64 [%0], %1;" ::"r"(remote + 16 * rank + 8), "d"(tp) : "memory");
+    asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote + 16 * rank), "f"(dh), "f"(dl),
+                 "f"(ph), "f"(pl)
+                 : "memory");
   }
   // All remote stores are done and visible to the leader; no CTA exits while
   // another may still write into its shared memory.
   cluster_sync_all();
   if (rank == 0 && threadIdx.x == 0) {
-    double td = 0.0, tp = 0.0;
+    float dh = 0.f, dl = 0.f, ph = 0.f, pl = 0.f;
     for (int r = 0; r < p.cs; ++r) {
-      td += slots[2 * r];
-      tp += slots[2 * r + 1];
+      const float4 v = slots[r];
+      ff_add(dh, dl, v.x);
+      dl += v.y;
+      ff_add(ph, pl, v.z);
+      pl += v.w;
     }
-    p.d_out[b * p.H + h] = float(sqrt(td) / (sqrt(tp) + double(p.eps)));
+    p.d_out[b * p.H + h] = sqrtf(dh + dl) / (sqrtf(ph + pl) + p.eps);
   }
 }
 
-// Clusters of cs CTAs of the S-stage kernel that can be resident at once on
+// The cluster kernels: (stages, unit bytes) = (8, 12 KB), (4, 12 KB), (8, 8 KB), (4, 8 KB).
+constexpr int CL_VARIANTS = 4;
+struct ClVariant {
+  int S, UB, threads, smem;
+  void (*fn)(ClusterParams);
+};
+inline const ClVariant& cl_variant(int i) {
+  static const ClVariant v[CL_VARIANTS] = {
+      {8, UNIT_BYTES, ClLayout<8, UNIT_BYTES>::THREADS, ClLayout<8, UNIT_BYTES>::ALLOC,
+       q_delta_cluster_kernel<8, UNIT_BYTES>},
+      {4, UNIT_BYTES, ClLayout<4, UNIT_BYTES>::THREADS, ClLayout<4, UNIT_BYTES>::ALLOC,
+       q_delta_cluster_kernel<4, UNIT_BYTES>},
+      {8, CL_UNIT_SMALL, ClLayout<8, CL_UNIT_SMALL>::THREADS, ClLayout<8, CL_UNIT_SMALL>::ALLOC,
+       q_delta_cluster_kernel<8, CL_UNIT_SMALL>},
+      {4, CL_UNIT_SMALL, ClLayout<4, CL_UNIT_SMALL>::THREADS, ClLayout<4, CL_UNIT_SMALL>::ALLOC,
+       q_delta_cluster_kernel<4, CL_UNIT_SMALL>},
+  };
+  return v[i];
+}
+
+// Clusters of cs CTAs of cluster variant vi that can be resident at once on
 // the current device (cached per device); -1 with the error set on failure.
 // Also raises the kernels' dynamic shared-memory limit once per device.
-int max_active_clusters(int S, int cs) {
+int max_active_clusters(int vi, int cs) {
   static std::mutex mu;
-  static int cache[64][2][CL_MAX_CS + 1];
+  static int cache[64][CL_VARIANTS][CL_MAX_CS + 1];
   static bool ready[64] = {false};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
@@ -437,18 +523,16 @@ int max_active_clusters(int S, int cs) {
   }
   std::lock_guard<std::mutex> lk(mu);
   if (!ready[dev]) {
-    cudaError_t e = cudaFuncSetAttribute(q_delta_cluster_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         ClLayout<8>::ALLOC);
-    if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(q_delta_cluster_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               ClLayout<4>::ALLOC);
-    for (int si = 0; si < 2 && e == cudaSuccess; ++si) {
+    cudaError_t e = cudaSuccess;
+    for (int i = 0; i < CL_VARIANTS && e == cudaSuccess; ++i)
+      e = cudaFuncSetAttribute(cl_variant(i).fn, cudaFuncAttributeMaxDynamicSharedMemorySize, cl_variant(i).smem);
+    for (int i = 0; i < CL_VARIANTS && e == cudaSuccess; ++i) {
       for (int c = 1; c <= CL_MAX_CS && e == cudaSuccess; ++c) {
         cudaLaunchConfig_t cfg;
         std::memset(&cfg, 0, sizeof(cfg));
         cfg.gridDim = dim3(c, 1, 1);
-        cfg.blockDim = dim3(si == 0 ? ClLayout<8>::THREADS : ClLayout<4>::THREADS, 1, 1);
-        cfg.dynamicSmemBytes = si == 0 ? ClLayout<8>::ALLOC : ClLayout<4>::ALLOC;
+        cfg.blockDim = dim3(cl_variant(i).threads, 1, 1);
+        cfg.dynamicSmemBytes = cl_variant(i).smem;
         cudaLaunchAttribute attr[1];
         attr[0].id = cudaLaunchAttributeClusterDimension;
         attr[0].val.clusterDim.x = c;
@@ -457,9 +541,8 @@ int max_active_clusters(int S, int cs) {
         cfg.attrs = attr;
         cfg.numAttrs = 1;
         int n = 0;
-        e = si == 0 ? cudaOccupancyMaxActiveClusters(&n, q_delta_cluster_kernel<8>, &cfg)
-                    : cudaOccupancyMaxActiveClusters(&n, q_delta_cluster_kernel<4>, &cfg);
-        cache[dev][si][c] = n;
+        e = cudaOccupancyMaxActiveClusters(&n, cl_variant(i).fn, &cfg);
+        cache[dev][i][c] = n;
       }
     }
     if (e != cudaSuccess) {
@@ -469,7 +552,7 @@ int max_active_clusters(int S, int cs) {
     }
     ready[dev] = true;
   }
-  return cache[dev][S == 8 ? 0 : 1][cs];
+  return cache[dev][vi][cs];
 }
 
 }  // namespace qd
@@ -479,7 +562,7 @@ extern "C" size_t refadapt_q_delta_workspace_size(int32_t B, int32_t H) {
   if (B < 1 || H < 1) return 0;
   const size_t bh = size_t(B) * size_t(H);
   const size_t counters = ((bh * sizeof(uint32_t)) + 255) / 256 * 256;
-  return counters + bh * ra::qd::MAX_SPLITS * 2 * sizeof(double);
+  return counters + bh * ra::qd::MAX_SPLITS * sizeof(float4);
 }
 
 namespace ra {
@@ -534,28 +617,33 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
     // run in one wave are candidates. Among those the one with the most bytes
     // in flight (CTAs x stages) wins. Taken when it occupies at least 60 % of
     // the CTAs the multi-block path would run (min(SMs, units)).
-    const int rows_per_unit = UNIT_BYTES / (2 * d);
+    const int ub = int64_t(n) * d * 2 <= CL_SMALL_SLAB_BYTES ? CL_UNIT_SMALL : UNIT_BYTES;
+    const int rows_per_unit = ub / (2 * d);
     const int per_slab = (n + rows_per_unit - 1) / rows_per_unit;
     const int64_t sms = num_sms();
-    int best_s = 0, best_cs = 0;
+    int best_v = -1, best_cs = 0;
     int64_t best_score = 0;
-    for (int S : {8, 4}) {
+    for (int vi = 0; vi < CL_VARIANTS; ++vi) {
+      const int S = cl_variant(vi).S;
+      if (cl_variant(vi).UB != ub) continue;
       for (int cs = 1; cs <= CL_MAX_CS && cs <= per_slab; ++cs) {
         if ((per_slab + cs - 1) / cs > CL_MAX_UNITS) continue;
-        const int fit = max_active_clusters(S, cs);
+        const int fit = max_active_clusters(vi, cs);
         if (fit < 0) return RA_ECUDA;
         if (bh > fit) continue;
         const int64_t score = int64_t(bh) * cs * S;
         if (score > best_score) {
           best_score = score;
-          best_s = S;
+          best_v = vi;
           best_cs = cs;
         }
       }
     }
-    const int64_t units_all = int64_t(bh) * per_slab;
+    // The multi-block path's units are 12 KB.
+    const int64_t units_all = int64_t(bh) * ((int64_t(n) * d * 2 + UNIT_BYTES - 1) / UNIT_BYTES);
     const int64_t ticket_ctas = units_all < sms ? units_all : sms;
-    if (best_s != 0 && double(bh) * best_cs >= 0.6 * double(ticket_ctas)) {
+    if (best_v >= 0 && double(bh) * best_cs >= 0.6 * double(ticket_ctas)) {
+      const ClVariant& cv = cl_variant(best_v);
       ClusterParams c;
       std::memset(&c, 0, sizeof(c));
       c.bulk = (q_cur->stride_n == d && q_prev->stride_n == d) ? 1 : 0;
@@ -580,8 +668,8 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
       cudaLaunchConfig_t cfg;
       std::memset(&cfg, 0, sizeof(cfg));
       cfg.gridDim = dim3(best_cs, H, B);
-      cfg.blockDim = dim3(best_s == 8 ? ClLayout<8>::THREADS : ClLayout<4>::THREADS, 1, 1);
-      cfg.dynamicSmemBytes = best_s == 8 ? ClLayout<8>::ALLOC : ClLayout<4>::ALLOC;
+      cfg.blockDim = dim3(cv.threads, 1, 1);
+      cfg.dynamicSmemBytes = cv.smem;
       cfg.stream = static_cast<cudaStream_t>(stream);
       cudaLaunchAttribute attr[2];
       attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -594,8 +682,7 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
       attr[1].val.programmaticStreamSerializationAllowed = 1;
       cfg.attrs = attr;
       cfg.numAttrs = 2;
-      const cudaError_t e = best_s == 8 ? cudaLaunchKernelEx(&cfg, q_delta_cluster_kernel<8>, c)
-                                        : cudaLaunchKernelEx(&cfg, q_delta_cluster_kernel<4>, c);
+      const cudaError_t e = cudaLaunchKernelEx(&cfg, cv.fn, c);
       if (e != cudaSuccess) {
         set_error("%s: cluster launch failed: %s", who, cudaGetErrorString(e));
         cudaGetLastError();
@@ -626,7 +713,7 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
   p.d_out = d_out;
   const size_t counters = ((size_t(bh) * sizeof(uint32_t)) + 255) / 256 * 256;
   p.counter = static_cast<uint32_t*>(workspace);
-  p.partial = reinterpret_cast<double*>(static_cast<char*>(workspace) + counters);
+  p.partial = reinterpret_cast<float4*>(static_cast<char*>(workspace) + counters);
   p.budget_ns = wait_budget_ns();
   p.bulk = (q_cur->stride_n == d && q_prev->stride_n == d) ? 1 : 0;
   p.base_c = static_cast<const char*>(q_cur->ptr);
@@ -689,7 +776,7 @@ namespace qd {
 
 constexpr int kNoAllocMaxBH = RA_Q_DELTA_NOALLOC_MAX_BH;
 constexpr size_t kNoAllocCounterBytes = ((size_t(kNoAllocMaxBH) * sizeof(uint32_t)) + 255) / 256 * 256;
-constexpr size_t kNoAllocBytes = kNoAllocCounterBytes + size_t(kNoAllocMaxBH) * MAX_SPLITS * 2 * sizeof(double);
+constexpr size_t kNoAllocBytes = kNoAllocCounterBytes + size_t(kNoAllocMaxBH) * MAX_SPLITS * sizeof(float4);
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoAllocBytes];
 

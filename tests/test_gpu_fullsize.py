@@ -26,10 +26,11 @@ def _role(X, wl, r, z):
     return X[z, :, :, o:o + wl.n[r], :]
 
 
-def _run_stack(wl, blocks):
+def _run_stack(wl, blocks, sample_stride=1):
     """Run the executor over `blocks` (indices into the workload's block
     stack, as a depth-reduced stack) for all steps; returns per (t, b) the
-    inputs, outputs, D, modes, gbar and mass partials as seen after the block."""
+    inputs, outputs, D, modes, gbar and mass partials as seen after the block.
+    sample_stride k > 1: D and M over the target rows 0, k, 2k, ..."""
     from paper_2609_32415_gb300 import Executor, roles_from_joint, synth
     sub = synth.Workload(**{**wl.__dict__})
     sub.n_blocks = len(blocks)
@@ -38,7 +39,7 @@ def _run_stack(wl, blocks):
     traj = synth.Trajectory(sub, device="cuda")
     ex = Executor(sub.n_blocks, sub.B, sub.H, sub.d, sub.n_text, sub.n_ref, sub.n_tgt, sub.theta,
                   sub.delta_max, sub.eps, mass_rows=sub.mass_rows, forced_boundary=sub.forced_boundary,
-                  bias=sub.bias, log_steps=sub.n_steps)
+                  bias=sub.bias, log_steps=sub.n_steps, sample_stride=sample_stride)
     rec = {}
     prev = {}
     for t in range(sub.n_steps):
@@ -50,7 +51,7 @@ def _run_stack(wl, blocks):
             torch.cuda.synchronize()
             rec[(t, b)] = {"X": X, "O": out, "D": ex.D[b].clone(), "mode": ex.modes[t, b].clone(),
                            "gbar": ex.gbar[t, b].clone(), "mass": ex.mass[b].clone(),
-                           "Xprev": prev.get(b)}
+                           "M": ex.M[t, b].clone(), "Xprev": prev.get(b)}
             prev[b] = X
         # keep only what later checks need
     ex.check()
@@ -179,3 +180,64 @@ def test_fullsize_depth_reduced_trajectory(cuda_ok):
             assert gm[:k] == [0] * k and gm[k + 1:] == [2] * (len(gm) - k - 1)
         else:
             assert gm == [0] * len(blocks)
+
+
+def test_fullsize_trajectory_on_oracle_mass(cuda_ok):
+    """Image-edit workload, depth-reduced stack {0, 1, 44, 45, 59}, all 8
+    steps, D and M over the sampled target rows 0, 16, 32, ... (256 of 4096):
+    at every (t, b) the oracle computes M (Eq. 4) for all 24 heads from the
+    keys the block executed (the reference keys of its last materialisation,
+    kept by the oracle's own bookkeeping of Eq. 11) and D (Eq. 1) on the same
+    rows; the GPU's M must agree within 2e-5 and its D within the Q-change
+    tolerance, and the oracle's controller, fed with the oracle's own D and M
+    only, must reproduce every decision."""
+    from paper_2609_32415_gb300 import synth
+    k = 16
+    wl = synth.make_workload("c2")
+    blocks = [0, 1, 44, 45, 59]
+    sub, rec = _run_stack(wl, blocks, sample_stride=k)
+    sc = 1.0 / math.sqrt(sub.d)
+    r0, r1 = sub.n_text, sub.n_text + sub.n_ref
+    nb = len(blocks)
+    gate = oracle.Gate(1, sub.theta, sub.delta_max, sub.forced_boundary)
+    a_b = [-1] * nb                      # the oracle's own materialisation step per block
+    m_prev = [None] * nb                 # the oracle's M of the previous step per block
+    m_prev_gate = [None] * nb
+    m_err = 0.0
+    for t in range(sub.n_steps):
+        gate.begin_step(t)
+        gm = [int(rec[(t, b)]["mode"][0]) for b in range(nb)]
+        for b in range(nb):
+            r = rec[(t, b)]
+            qt = _wide(_role(r["X"], sub, "tgt", 0)[0, :, ::k])            # [H, 256, d]
+            if t >= 1:
+                qp = _wide(_role(r["Xprev"], sub, "tgt", 0)[0, :, ::k])
+                D = oracle.q_change(qt, qp, sub.eps)                       # [H]
+                got = r["D"][0].double().cpu().numpy()
+                assert (np.abs(got - D) / D).max() <= D_REL, (t, b)
+                m, _ = gate.decide(t, b, D[None], m_prev[b][None],
+                                   tie=lambda tt, bb, s: gm[bb] == 1, tie_band=TIE_BAND)
+            else:
+                m, _ = gate.decide(t, b)
+            assert m[0] == gm[b], (t, b, m, gm)
+            if m[0] in (2, 3):
+                a_b[b] = t
+            Xk = r["X"] if m[0] in (2, 3) else rec[(a_b[b], b)]["X"]
+            keys = np.concatenate([_wide(_role(r["X"], sub, "text", 1)[0]), _wide(_role(Xk, sub, "ref", 1)[0]),
+                                   _wide(_role(r["X"], sub, "tgt", 1)[0])], axis=1)
+            vals = np.concatenate([_wide(_role(r["X"], sub, "text", 2)[0]), _wide(_role(Xk, sub, "ref", 2)[0]),
+                                   _wide(_role(r["X"], sub, "tgt", 2)[0])], axis=1)
+            _, rm = oracle.joint_attention(qt, keys, vals, sc, ref_range=(r0, r1), want_o=False)
+            M = oracle.exposure(rm)                                         # [H]
+            # the GPU's M of this step's attention: its mass partials over the
+            # sampled rows (text tiles hold zero), as the next step's gate sums them
+            got = r["mass"][0].double().sum(-1).cpu().numpy() / qt.shape[1]
+            err = np.abs(got - M).max()
+            m_err = max(m_err, err)
+            assert err <= 2e-5, (t, b, err)
+            m_prev[b] = M
+            if t >= 1:   # the gate of step t read M of step t - 1 (its m_out)
+                assert np.abs(r["M"][0].double().cpu().numpy() - m_prev_gate[b]).max() <= 2e-5, (t, b)
+            m_prev_gate[b] = M
+    gm_all = [[int(rec[(t, b)]["mode"][0]) for b in range(nb)] for t in range(sub.n_steps)]
+    assert any(0 in row for row in gm_all[1:]) and any(1 in row for row in gm_all[1:]), gm_all

@@ -24,11 +24,11 @@ def _d(q_cur, q_prev, eps=1e-6, ws=None):
                                      (1, 24, 16380, 128), (2, 20, 700, 128), (8, 25, 130, 64),
                                      (1, 1, 100000, 128), (2, 1, 200000, 64), (1, 2, 20000, 128)])
 def test_q_delta_matches_oracle(cuda_ok, B, H, n, d):
-    """On a 152-SM GB300: (1, 24, ...) runs clusters of 5 CTAs with 8
-    stages, (2, 20, ...) clusters of 3 with 8 stages, (8, 25, ...) single-CTA
-    clusters with 4 stages; the last three (slabs too long for a cluster, or
-    too few slabs to fill the GPU) take the workspace path with per-slab
-    tickets."""
+    """The shapes span both unit sizes of the cluster path (8 KB units for
+    slabs up to 2 MB, 12 KB beyond: (1, 24, 16380, 128)), several cluster
+    sizes and both stage counts, ragged last units, and, in the last three
+    (slabs too long for a cluster, or too few slabs to fill the GPU), the
+    workspace path with per-slab tickets."""
     g = torch.Generator().manual_seed(n + d)
     prev = (torch.randn((B, H, n, d), generator=g) / d ** 0.5).to(torch.bfloat16)
     cur = (prev.float() + 0.3 * torch.randn((B, H, n, d), generator=g) / d ** 0.5).to(torch.bfloat16)
