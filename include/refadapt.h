@@ -152,7 +152,7 @@ int32_t refadapt_mass_partial_len(int32_t n_text, int32_t n_tgt);
  *
  * Each slab (one sample and head) is reduced by one thread-block cluster of
  * up to 8 CTAs through distributed shared memory, leaving the workspace
- * untouched, when a slab has at most 8 x 256 units of 12 KB per tensor
+ * untouched, when a slab has at most 8 x 384 units of 8 KB per tensor
  * (n <= 98304 rows at d = 128, 196608 at d = 64), all B * H clusters fit on
  * the GPU at once, and they fill at least 60 % of the SMs (or of the units,
  * for tiny inputs). Otherwise a

@@ -1,8 +1,9 @@
 // refadapt_q_delta: relative L2 change of the target query per (sample, head),
 // D = ||q_t - q_{t-1}||_F / (||q_{t-1}||_F + eps)   (paper Eq. 1, Sec. 4).
 //
-// HBM-bound streaming reduction. Work is cut into units of 12 KB per tensor
-// (48 rows at d = 128, 96 rows at d = 64) of one (sample, head) slab. When
+// HBM-bound streaming reduction. Work is cut into units of one (sample,
+// head) slab: 8 KB per tensor on the cluster path, 12 KB on the multi-block
+// path (32 / 48 rows at d = 128, 64 / 96 at d = 64). When
 // both tensors' rows are contiguous within a slab (stride_n == d) a unit is
 // one 1-D bulk copy of its bytes (the slab's last unit is shorter); otherwise
 // it is a 2-D TMA tensor load (any row strides; rows past the slab end arrive
@@ -20,8 +21,8 @@
 //
 // Cluster path (used when the slabs fit clusters that fill the GPU): one
 // cluster of up to 8 CTAs per (sample, head) slab, each CTA streaming its
-// contiguous share of the slab's units through an 8-stage ring (one CTA per
-// SM) or a 4-stage ring (two per SM), whichever fills the SMs better; every
+// contiguous share of the slab's units through a 12-stage ring (one CTA per
+// SM) or a 6-stage ring (two per SM), whichever keeps more bytes in flight; every
 // CTA stores its sums into the cluster leader's shared memory (distributed
 // shared memory) and, after one cluster barrier, the leader adds them in rank
 // order and writes D. No global atomics, fences or workspace: the reduction
@@ -279,14 +280,15 @@ __global__ void __launch_bounds__(THREADS, 1) q_delta_kernel(const __grid_consta
 
 // ---------------------------------------------------------------- cluster path
 constexpr int CL_MAX_CS = 8;       // CTAs per cluster (portable limit)
-constexpr int CL_MAX_UNITS = 256;  // units per CTA (longer slabs take the multi-block path)
+constexpr int CL_MAX_UNITS = 384;  // units per CTA (longer slabs take the multi-block path)
 
-// Units of the cluster path: 8 KB per tensor for slabs of up to 2 MB, 12 KB
-// for longer ones. On a short read (image edit: 24 slabs of 1 MB) the smaller
-// first wave of requests and the finer split make a launch 2 % shorter; on a
-// long one (video: 24 slabs of 4.2 MB) the larger units stream 3 % faster.
-constexpr int CL_UNIT_SMALL = 8192;
-constexpr int64_t CL_SMALL_SLAB_BYTES = int64_t(2) << 20;
+// Units of the cluster path: 8 KB per tensor (32 rows at d = 128, 64 at d = 64).
+// What sets a short read's time is how many units each SM has in flight and
+// how many warps drain them: 12 stages of 8 KB (192 KB, 12 consumer warps)
+// read the image-edit target query (24 slabs of 1 MB) in 9.8 us and the video
+// one (24 slabs of 4.2 MB) in 31.4 us, against 10.7 and 31.9 us for 8 stages
+// of 12 KB over the same 192 KB, and 13.2 us for 6 stages of 8 KB.
+constexpr int CL_UNIT_BYTES = 8192;
 
 // Shared-memory layout of a cluster CTA with S stages of UB-byte units per
 // tensor (stage s belongs to consumer warp s; warp S is the producer).
@@ -300,9 +302,8 @@ struct ClLayout {
   static constexpr int BYTES = OFF_SLOTS + CL_MAX_CS * 16;
   static constexpr int ALLOC = BYTES + 1024;
 };
-static_assert(ClLayout<8, UNIT_BYTES>::ALLOC <= 232448, "shared memory budget");
-static_assert(2 * ClLayout<4, UNIT_BYTES>::ALLOC <= 232448, "two 4-stage CTAs per SM");
-static_assert(ClLayout<8, CL_UNIT_SMALL>::ALLOC <= 232448, "shared memory budget");
+static_assert(ClLayout<12, CL_UNIT_BYTES>::ALLOC <= 232448, "shared memory budget");
+static_assert(2 * ClLayout<6, CL_UNIT_BYTES>::ALLOC <= 232448, "two 6-stage CTAs per SM");
 
 struct ClusterParams {
   CUtensorMap tm_c, tm_p;
@@ -489,22 +490,18 @@ __global__ void __launch_bounds__(ClLayout<S, UB>::THREADS)
   }
 }
 
-// The cluster kernels: (stages, unit bytes) = (8, 12 KB), (4, 12 KB), (8, 8 KB), (4, 8 KB).
-constexpr int CL_VARIANTS = 4;
+// The cluster kernels: 12 stages (one CTA per SM) or 6 stages (two per SM).
+constexpr int CL_VARIANTS = 2;
 struct ClVariant {
-  int S, UB, threads, smem;
+  int S, threads, smem;
   void (*fn)(ClusterParams);
 };
 inline const ClVariant& cl_variant(int i) {
   static const ClVariant v[CL_VARIANTS] = {
-      {8, UNIT_BYTES, ClLayout<8, UNIT_BYTES>::THREADS, ClLayout<8, UNIT_BYTES>::ALLOC,
-       q_delta_cluster_kernel<8, UNIT_BYTES>},
-      {4, UNIT_BYTES, ClLayout<4, UNIT_BYTES>::THREADS, ClLayout<4, UNIT_BYTES>::ALLOC,
-       q_delta_cluster_kernel<4, UNIT_BYTES>},
-      {8, CL_UNIT_SMALL, ClLayout<8, CL_UNIT_SMALL>::THREADS, ClLayout<8, CL_UNIT_SMALL>::ALLOC,
-       q_delta_cluster_kernel<8, CL_UNIT_SMALL>},
-      {4, CL_UNIT_SMALL, ClLayout<4, CL_UNIT_SMALL>::THREADS, ClLayout<4, CL_UNIT_SMALL>::ALLOC,
-       q_delta_cluster_kernel<4, CL_UNIT_SMALL>},
+      {12, ClLayout<12, CL_UNIT_BYTES>::THREADS, ClLayout<12, CL_UNIT_BYTES>::ALLOC,
+       q_delta_cluster_kernel<12, CL_UNIT_BYTES>},
+      {6, ClLayout<6, CL_UNIT_BYTES>::THREADS, ClLayout<6, CL_UNIT_BYTES>::ALLOC,
+       q_delta_cluster_kernel<6, CL_UNIT_BYTES>},
   };
   return v[i];
 }
@@ -610,22 +607,20 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
   const int n = q_cur->n;
   const int bh = B * H;
   {
-    // Cluster path. Stages S = 8 (one CTA per SM, 192 KB in flight) or S = 4
-    // (two CTAs per SM); cluster size cs <= 8. Clusters live inside one GPC,
+    // Cluster path. Stages S = 12 (one CTA per SM, 192 KB in flight) or
+    // S = 6 (two CTAs per SM); cluster size cs <= 8. Clusters live inside one GPC,
     // so how many fit at once depends on the GPU's floorplan: the runtime's
     // occupancy query says, and only configurations whose B * H clusters all
     // run in one wave are candidates. Among those the one with the most bytes
     // in flight (CTAs x stages) wins. Taken when it occupies at least 60 % of
     // the CTAs the multi-block path would run (min(SMs, units)).
-    const int ub = int64_t(n) * d * 2 <= CL_SMALL_SLAB_BYTES ? CL_UNIT_SMALL : UNIT_BYTES;
-    const int rows_per_unit = ub / (2 * d);
+    const int rows_per_unit = CL_UNIT_BYTES / (2 * d);
     const int per_slab = (n + rows_per_unit - 1) / rows_per_unit;
     const int64_t sms = num_sms();
     int best_v = -1, best_cs = 0;
     int64_t best_score = 0;
     for (int vi = 0; vi < CL_VARIANTS; ++vi) {
       const int S = cl_variant(vi).S;
-      if (cl_variant(vi).UB != ub) continue;
       for (int cs = 1; cs <= CL_MAX_CS && cs <= per_slab; ++cs) {
         if ((per_slab + cs - 1) / cs > CL_MAX_UNITS) continue;
         const int fit = max_active_clusters(vi, cs);
