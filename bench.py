@@ -106,9 +106,12 @@ def source_hash(*rel):
 ATTN_SOURCES = ("paper_2609_32415_gb300/csrc/joint_attn.cu", "paper_2609_32415_gb300/csrc/tc_ptx.cuh")
 
 
-def recorded_traffic(config):
+def recorded_traffic(config, modes=None):
     """DRAM bytes per attention launch from the committed ncu summary, or None
-    when the kernel source changed since the counters were taken."""
+    when the kernel source changed since the counters were taken. A record with
+    separate refresh and reuse launches is averaged over the timed launches'
+    modes (`modes`: one list of per-sample modes per launch; a launch counts as
+    refresh when any sample materialises)."""
     path = os.path.join(ROOT, "profiles", "attn_traffic.json")
     try:
         with open(path) as f:
@@ -117,7 +120,17 @@ def recorded_traffic(config):
         return None
     if rec.get("source_hash") != source_hash(*ATTN_SOURCES):
         return None
-    return rec.get("per_launch", {}).get(config)
+    r = rec.get("per_launch", {}).get(config)
+    if r is None or "bytes" in r:
+        return r
+    if not modes or "refresh" not in r or "reuse" not in r:
+        return None
+    n_ref = sum(1 for m in modes if any(int(x) != 0 for x in m))
+    n_reu = len(modes) - n_ref
+    out = {"bytes": int(round((n_ref * r["refresh"]["bytes"] + n_reu * r["reuse"]["bytes"]) / len(modes))),
+           "mix": {"refresh_launches": n_ref, "reuse_launches": n_reu},
+           "refresh": r["refresh"], "reuse": r["reuse"], "capture": r.get("capture")}
+    return out
 
 
 class Clocks:
@@ -352,6 +365,7 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
         res["attn_ms_sum_of_launches"] = ms_sum
         res["attn_flops"] = flops
         res["attn_launches"] = len(ev)
+        res["attn_launch_tb"] = [(t, b) for (t, b, _) in ev]
     del ex
     return res
 
@@ -868,7 +882,7 @@ def main_ours(args):
             dist.destroy_process_group()
         return
     attn_tflops = main["attn_flops"] / (main["attn_ms"] * 1e-3) / 1e12
-    traffic = recorded_traffic(args.config)
+    traffic = recorded_traffic(args.config, [list(main["modes"][t, b]) for t, b in main["attn_launch_tb"]])
     per_launch_flops = main["attn_flops"] / main["attn_launches"]
     qsum = q_delta_summary(qd, peaks)
     if qd_long is not None:

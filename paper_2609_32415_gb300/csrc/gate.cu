@@ -51,11 +51,21 @@ __global__ void init_kernel(ra_state* st, int32_t B) {
   }
 }
 
+// (hi, lo) += x with the rounding error of the addition kept in lo (TwoSum;
+// the value is hi + lo). The sums stay off the FP64 pipe, which is narrow on
+// this GPU, with about the accuracy of fp64 over these few terms.
+__device__ __forceinline__ void ff_add(float& hi, float& lo, float x) {
+  const float s = hi + x;
+  const float v = s - hi;
+  lo += (hi - (s - v)) + (x - v);
+  hi = s;
+}
+
 // One CTA. Warps compute M_{t-1,b,h} for every (sample, head) from the mass
-// partials (lane-strided sums, then a butterfly: fixed order, fp64) into
-// shared memory; then thread s takes sample s through the decision.
+// partials (lane-strided two-float sums, then a fixed tree over the lanes)
+// into shared memory; then thread s takes sample s through the decision.
 __global__ void __launch_bounds__(THREADS) gate_kernel(const Params p) {
-  extern __shared__ double m_sh[];  // [B * H]
+  extern __shared__ float m_sh[];  // [B * H]
   ra_state* st = p.st;
   int32_t* reactivated = reinterpret_cast<int32_t*>(st + 1);
   int32_t* boundary = reactivated + p.B;
@@ -78,17 +88,21 @@ __global__ void __launch_bounds__(THREADS) gate_kernel(const Params p) {
     full_step = st->full_step;
   }
   for (int sh = warp; sh < p.B * p.H; sh += nwarps) {
-    double acc = 0.0;
+    float hi = 0.f, lo = 0.f;
     if (p.mp) {
       const float* row = p.mp + int64_t(sh) * p.mpl;
-      for (int i = lane; i < p.mpl; i += 32) acc += double(row[i]);
+      for (int i = lane; i < p.mpl; i += 32) ff_add(hi, lo, row[i]);
 #pragma unroll
-      for (int o = 16; o > 0; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+      for (int o = 16; o > 0; o >>= 1) {
+        const float xh = __shfl_down_sync(0xffffffffu, hi, o), xl = __shfl_down_sync(0xffffffffu, lo, o);
+        ff_add(hi, lo, xh);
+        lo += xl;
+      }
     }
     if (lane == 0) {
-      const double m = acc / double(p.mass_rows_count);
+      const float m = (hi + lo) / float(p.mass_rows_count);
       m_sh[sh] = m;
-      if (p.m_out && p.mp) p.m_out[sh] = float(m);
+      if (p.m_out && p.mp) p.m_out[sh] = m;
     }
   }
   __syncthreads();
@@ -98,14 +112,24 @@ __global__ void __launch_bounds__(THREADS) gate_kernel(const Params p) {
       boundary[s] = -1;
     }
     const bool have = (p.t >= 1) && p.qd && p.mp;
-    double gsum = 0.0;
+    float ghi = 0.f, glo = 0.f;
     if (have) {
       for (int h = 0; h < p.H; ++h) {
-        const double dh = double(p.qd[s * p.H + h]), mh = m_sh[s * p.H + h];
-        gsum += (p.cue == RA_CUE_CHANGE) ? dh : (p.cue == RA_CUE_EXPOSURE) ? mh : dh * mh;
+        const float dh = p.qd[s * p.H + h], mh = m_sh[s * p.H + h];
+        if (p.cue == RA_CUE_CHANGE) {
+          ff_add(ghi, glo, dh);
+        } else if (p.cue == RA_CUE_EXPOSURE) {
+          ff_add(ghi, glo, mh);
+        } else {
+          // the product's rounding error joins lo (exact by one fma)
+          const float g = dh * mh;
+          ff_add(ghi, glo, g);
+          glo += fmaf(dh, mh, -g);
+        }
       }
     }
-    const double gbar = have ? gsum / double(p.H) : NAN;
+    // The comparison with theta (a double) is made in fp64 on hi + lo.
+    const double gbar = have ? (double(ghi) + double(glo)) / double(p.H) : NAN;
     if (p.gbar_out) p.gbar_out[s] = float(gbar);
     int32_t mode;
     if (full_step) {
@@ -197,7 +221,7 @@ extern "C" ra_status refadapt_gate(const ra_gate_args* a, void* stream) {
   p.mode_out = a->mode_out;
   p.gbar_out = a->gbar_out;
   p.m_out = a->m_out;
-  const size_t sh_bytes = size_t(a->B) * a->H * sizeof(double);
+  const size_t sh_bytes = size_t(a->B) * a->H * sizeof(float);
   gate::gate_kernel<<<1, gate::THREADS, sh_bytes, static_cast<cudaStream_t>(stream)>>>(p);
   return launch_status("refadapt_gate");
 }
