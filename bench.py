@@ -398,6 +398,33 @@ def time_graphs(wl, inputs, warmup, steps):
     return {"ms_per_step": e0.elapsed_time(e1) / steps, "modes": modes}
 
 
+class PinnedArena:
+    """Page-locked host memory handed out from a few large blocks of torch's
+    pinned allocator. That allocator rounds every request up to a power of
+    two, so one 612 MB buffer per (step, block) would pin 1 GiB each (the
+    video trajectory: 171 GB of the host's 199 GB); blocks of a power-of-two
+    size are used whole and sub-allocated in order instead."""
+
+    def __init__(self, total_bytes, largest_bytes, block_bytes=16 << 30):
+        import torch
+        self.torch = torch
+        need = max(int(total_bytes), int(largest_bytes), 1)
+        size = 1 << (need - 1).bit_length()
+        self.block = min(size, max(block_bytes, 1 << (int(largest_bytes) - 1).bit_length()))
+        self.blocks, self.used = [], self.block
+        self.pinned = 0
+
+    def take(self, numel, dtype):
+        nbytes = (numel * self.torch.empty((), dtype=dtype).element_size() + 511) // 512 * 512
+        if self.used + nbytes > self.block:
+            self.blocks.append(self.torch.empty(self.block, dtype=self.torch.uint8, pin_memory=True))
+            self.pinned += self.block
+            self.used = 0
+        out = self.blocks[-1][self.used:self.used + numel * self.torch.empty((), dtype=dtype).element_size()]
+        self.used += nbytes
+        return out.view(dtype)
+
+
 def time_e2e(wl, inputs, warmup, steps):
     """Same steps through the public API with host-resident inputs and results.
 
@@ -444,10 +471,15 @@ def time_e2e(wl, inputs, warmup, steps):
 
     o_base, o_ref = size["tq"], size["tq"] + size["base"]
     # Page-locked host trajectory (cudaHostAlloc through torch's pinned
-    # allocator), written by the CPU: each block's bytes go device -> a
-    # staging buffer, then a host memcpy into the block's own buffer.
+    # allocator, sub-allocated from large blocks), written by the CPU: each
+    # block's bytes go device -> a staging buffer, then a host memcpy into the
+    # block's own buffer.
+    out_elems = sum(math.prod(shape[r]) for r in ROLES)
+    arena = PinnedArena(2 * (T * nb * per_block + nb * out_elems), 2 * per_block)
     stage = torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True)
     stage_v = {"tq": views(stage, 0, "tq"), "base": views(stage, o_base, "base"), "ref": views(stage, o_ref, "ref")}
+    # Page-locked host outputs, one set per block (each step overwrites them).
+    hout = [{r: arena.take(math.prod(shape[r]), torch.bfloat16).view(shape[r]) for r in ROLES} for _ in range(nb)]
     bufs, host = [], []
     for t in range(T):
         brow, hrow = [], []
@@ -456,15 +488,13 @@ def time_e2e(wl, inputs, warmup, steps):
             for kind in stage_v:
                 for (z, r), h in stage_v[kind].items():
                     h.copy_(X[z, :, :, off[r]:off[r] + wl.n[r], :])
-            buf = torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True)
+            buf = arena.take(per_block, torch.bfloat16)
             buf.copy_(stage)
             brow.append(buf)
             hrow.append({k: buf[o:o + size[k]] for k, o in (("tq", 0), ("base", o_base), ("ref", o_ref))})
         bufs.append(brow)
         host.append(hrow)
     del stage, stage_v
-    # Page-locked host outputs, one set per block (each step overwrites them).
-    hout = [{r: torch.empty(shape[r], dtype=torch.bfloat16, pin_memory=True) for r in ROLES} for _ in range(nb)]
     torch.cuda.synchronize()
     dev = torch.device("cuda")
     # Device staging: each block's target Q for the current and the previous
@@ -599,7 +629,8 @@ def time_e2e(wl, inputs, warmup, steps):
     torch.cuda.synchronize()
     ms, per_step, h2d_b, d2h_b = timed(T + warmup, steps)
     ex.check()
-    del host, slots, slot_v, osl, tq, ex, bufs, hout
+    pinned_gb = arena.pinned / 1e9
+    del host, slots, slot_v, osl, tq, ex, bufs, hout, arena
     pipeline = ("per step: the step's gates first (every block's target Q copied during the previous step), one "
                 "read of the modes, then per block text Q/K/V + target K/V and reference Q/K/V only where a "
                 "sample materialises, plus the next step's target Q; every executed output row (text and target, "
@@ -607,8 +638,9 @@ def time_e2e(wl, inputs, warmup, steps):
                 "mean over the timed steps")
     return {"value": ms, "unit": "ms/step", "per_step_ms": per_step, "h2d_bytes_per_step": h2d_b,
             "d2h_bytes_per_step": d2h_b,
-            "host_buffers": "pinned (cudaHostAlloc), one per (step, block) and one output set per block, written "
-                            "by the CPU; timed after the first trajectory over them and %d warm-up steps" % warmup,
+            "host_buffers": "pinned (cudaHostAlloc, %.1f GB in 16 GiB blocks), one buffer per (step, block) and "
+                            "one output set per block, written by the CPU; timed after the first trajectory over "
+                            "them and %d warm-up steps" % (pinned_gb, warmup),
             "pipeline": pipeline,
             "first_use": {"value": first_ms, "unit": "ms/step", "per_step_ms": first_steps,
                           "h2d_bytes_per_step": first_h2d, "d2h_bytes_per_step": first_d2h,
