@@ -425,7 +425,7 @@ class PinnedArena:
         return out.view(dtype)
 
 
-def time_e2e(wl, inputs, warmup, steps):
+def time_e2e(wl, inputs, warmup, steps, keep=None):
     """Same steps through the public API with host-resident inputs and results.
 
     Host side: one page-locked buffer per (step, block) with that block's
@@ -450,7 +450,11 @@ def time_e2e(wl, inputs, warmup, steps):
     the host buffers were written (no untimed pass over them: what a caller's
     first trajectory sees, with the device's translations of freshly pinned
     host memory still cold), then, after `warmup` more steps, `steps` timed
-    steps (steady state)."""
+    steps (steady state).
+
+    With `keep` (a list) nothing is timed: one trajectory runs step by step
+    through the same pipeline and `keep` receives, per step, the modes read
+    by the host and a copy of every block's host outputs (for tests)."""
     import torch
     from paper_2609_32415_gb300 import Executor
     T, nb = wl.n_steps, wl.n_blocks
@@ -623,6 +627,15 @@ def time_e2e(wl, inputs, warmup, steps):
                 int(h2d[0] // k), int(d2h[0] // k))
 
     torch.cuda.synchronize()
+    if keep is not None:
+        for i in range(T):
+            one_step(seq[i], counter, seq[i + 1])
+            torch.cuda.synchronize()
+            keep.append({"t": seq[i], "modes": modes_host.clone(),
+                         "out": [{r: hout[b][r].clone() for r in ROLES} for b in range(nb)]})
+        ex.check()
+        del host, slots, slot_v, osl, tq, ex, bufs, hout, arena
+        return keep
     first_ms, first_steps, first_h2d, first_d2h = timed(0, T)
     for i in range(warmup):
         one_step(seq[T + i], counter, seq[T + i + 1])
