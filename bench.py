@@ -398,6 +398,22 @@ def time_graphs(wl, inputs, warmup, steps):
     return {"ms_per_step": e0.elapsed_time(e1) / steps, "modes": modes}
 
 
+def host_memory_share():
+    """Bytes of host memory available to this rank: MemAvailable divided by the
+    ranks on this node (LOCAL_WORLD_SIZE); None when it cannot be read."""
+    try:
+        with open("/proc/meminfo") as f:
+            for ln in f:
+                if ln.startswith("MemAvailable:"):
+                    avail = int(ln.split()[1]) * 1024
+                    break
+            else:
+                return None
+    except OSError:
+        return None
+    return avail // max(1, int(os.environ.get("LOCAL_WORLD_SIZE", "1")))
+
+
 class PinnedArena:
     """Page-locked host memory handed out from a few large blocks of torch's
     pinned allocator. That allocator rounds every request up to a power of
@@ -479,7 +495,12 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
     # block's bytes go device -> a staging buffer, then a host memcpy into the
     # block's own buffer.
     out_elems = sum(math.prod(shape[r]) for r in ROLES)
-    arena = PinnedArena(2 * (T * nb * per_block + nb * out_elems), 2 * per_block)
+    need = 2 * (T * nb * per_block + nb * out_elems)
+    share = host_memory_share()
+    if share is not None and need > 0.8 * share:
+        raise RuntimeError("host memory: the e2e trajectory needs %.1f GB pinned per rank, %.1f GB available to this "
+                           "rank" % (need / 1e9, share / 1e9))
+    arena = PinnedArena(need, 2 * per_block)
     stage = torch.empty(per_block, dtype=torch.bfloat16, pin_memory=True)
     stage_v = {"tq": views(stage, 0, "tq"), "base": views(stage, o_base, "base"), "ref": views(stage, o_ref, "ref")}
     # Page-locked host outputs, one set per block (each step overwrites them).

@@ -17,11 +17,11 @@ void clear_error();
 uint64_t wait_budget_ns();
 int num_sms();  // of the current device (cached per device)
 
-// Unique id of the CUDA context current in the calling thread, after making
-// sure the current device's primary context exists; 0 when the driver cannot
-// say. A context torn down (cudaDeviceReset) and created again gets a new id,
-// so state that belongs to a context (device addresses of module symbols) is
-// keyed by it.
+// Unique id of the CUDA context current in the calling thread; 0 when none is
+// current yet or the driver cannot say. Changes nothing (no context is made
+// current or created). A context torn down (cudaDeviceReset) and created
+// again gets a new id, so state that belongs to a context (device addresses
+// of module symbols) is keyed by it.
 uint64_t current_context_id();
 
 // Raises `func`'s dynamic shared-memory limit to `bytes` on the current

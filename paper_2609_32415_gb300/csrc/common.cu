@@ -93,13 +93,6 @@ uint64_t current_context_id() {
       get_id = reinterpret_cast<GetIdFn>(ptr);
   });
   if (!get_current || !get_id) return 0;
-  int dev = 0;
-  // cudaSetDevice on the current device makes its primary context current
-  // (and creates it) when the runtime has not done so yet.
-  if (cudaGetDevice(&dev) != cudaSuccess || cudaSetDevice(dev) != cudaSuccess) {
-    cudaGetLastError();
-    return 0;
-  }
   CUcontext ctx = nullptr;
   unsigned long long id = 0;
   if (get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr || get_id(ctx, &id) != CUDA_SUCCESS) return 0;

@@ -792,21 +792,21 @@ void* noalloc_scratch() {
     set_error("refadapt_q_delta_noalloc: no usable current device");
     return nullptr;
   }
-  const uint64_t ctx = current_context_id();  // 0: unknown, look the address up every call
   std::lock_guard<std::mutex> lk(g_noalloc_mu);
   NoAllocSlot& slot = g_noalloc[dev];
-  if (ctx == 0 || slot.ctx_id != ctx || slot.ptr == nullptr) {
-    void* ptr = nullptr;
-    const cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
-    if (e != cudaSuccess || ptr == nullptr) {
-      cudaGetLastError();
-      set_error("refadapt_q_delta_noalloc: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
-      return nullptr;
-    }
-    slot.ctx_id = ctx;
-    slot.ptr = ptr;
+  const uint64_t ctx = current_context_id();  // 0: no context yet, or unknown
+  if (ctx != 0 && slot.ctx_id == ctx && slot.ptr != nullptr) return slot.ptr;
+  // The lookup makes the device's primary context current when no context is.
+  void* ptr = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&ptr, g_noalloc_scratch);
+  if (e != cudaSuccess || ptr == nullptr) {
+    cudaGetLastError();
+    set_error("refadapt_q_delta_noalloc: cudaGetSymbolAddress failed: %s", cudaGetErrorString(e));
+    return nullptr;
   }
-  return slot.ptr;
+  slot.ctx_id = current_context_id();  // 0 (unknown): looked up again on the next call
+  slot.ptr = ptr;
+  return ptr;
 }
 
 }  // namespace qd

@@ -51,3 +51,27 @@ def test_cache_update_empty_reference(cuda_ok):
     api.refadapt_ref_cache_update(e, e, e, e, torch.tensor([2], dtype=torch.int32, device="cuda"), 4, a_b)
     torch.cuda.synchronize()
     assert a_b.item() == 4
+
+
+def test_cache_update_bulk_path_long_slabs(cuda_ok):
+    """Contiguous slabs (the executor's layout) take the bulk-copy path: video-
+    sized reference slabs (16,380 rows x 24 heads), so every CTA streams many
+    32 KB chunks through its ring, plus a hidden-state-like third tensor of one
+    3072-wide row per token; copied bit for bit for the materialising sample
+    only, a_b stamped for it only."""
+    from paper_2609_32415_gb300 import api
+    B, H, n, d, C = 2, 24, 16380, 128, 3072
+    g = torch.Generator(device="cuda").manual_seed(11)
+    src = [torch.randn((B, H, n, d), generator=g, device="cuda").to(torch.bfloat16) for _ in range(2)]
+    dst = [torch.zeros((B, H, n, d), dtype=torch.bfloat16, device="cuda") for _ in range(2)]
+    xs = torch.randn((B, 1, n, C), generator=g, device="cuda").to(torch.bfloat16)
+    xd = torch.zeros_like(xs)
+    mode = torch.tensor([2, 0], dtype=torch.int32, device="cuda")
+    a_b = torch.full((B,), -1, dtype=torch.int32, device="cuda")
+    api.refadapt_ref_cache_update(src[0], src[1], dst[0], dst[1], mode, 3, a_b, x_src=xs, x_cache=xd)
+    torch.cuda.synchronize()
+    assert a_b.tolist() == [3, -1]
+    for i in range(2):
+        assert torch.equal(dst[i][0], src[i][0])
+        assert torch.count_nonzero(dst[i][1]) == 0
+    assert torch.equal(xd[0], xs[0]) and torch.count_nonzero(xd[1]) == 0
