@@ -234,20 +234,36 @@ __device__ __forceinline__ void epilogue_tile(const Params& p, const Tile& tl, i
     }
   } else {
     const int64_t orow = int64_t(tl.s) * sg.out_ss + int64_t(valid ? r : 0) * sg.out_sr;
+    // RESID: the row's residual for the next 32 columns is loaded while the
+    // current 32 are computed (one global-load latency per tile, not per chunk).
+    const bool resid = p.epi == RA_EPI_RESID && valid;
+    const uint4* rrow = resid ? reinterpret_cast<const uint4*>(sg.resid + int64_t(tl.s) * sg.res_ss +
+                                                               int64_t(r) * sg.res_sr + tl.n0)
+                              : nullptr;
+    uint4 rnext[4];
+    if (resid) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) rnext[q] = rrow[q];
+    }
     for (int c0 = 0; c0 < BN; c0 += 32) {
       const int n = tl.n0 + c0;
+      uint4 rcur[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) rcur[q] = rnext[q];
+      if (resid && c0 + 32 < BN) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) rnext[q] = rrow[(c0 + 32) / 8 + q];
+      }
       float x[32];
       load_acc(base + c0, sg.bias, n, x);
       if (p.epi == RA_EPI_GELU) {
 #pragma unroll
         for (int j = 0; j < 32; ++j) x[j] = gelu_tanh(x[j]);
-      } else if (p.epi == RA_EPI_RESID && valid) {
-        const uint4* rp = reinterpret_cast<const uint4*>(sg.resid + int64_t(tl.s) * sg.res_ss +
-                                                         int64_t(r) * sg.res_sr + n);
+      } else if (resid) {
         const float4* gp = reinterpret_cast<const float4*>(sg.gate + int64_t(tl.s) * sg.gate_ss + n);
 #pragma unroll
         for (int q = 0; q < 4; ++q) {
-          const uint4 rv = rp[q];
+          const uint4 rv = rcur[q];
           const uint32_t w4[4] = {rv.x, rv.y, rv.z, rv.w};
           const float4 g0 = __ldg(gp + 2 * q), g1 = __ldg(gp + 2 * q + 1);
           const float gv[8] = {g0.x, g0.y, g0.z, g0.w, g1.x, g1.y, g1.z, g1.w};
