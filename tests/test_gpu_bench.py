@@ -1,0 +1,38 @@
+"""bench.py end to end on the small single-block workload: one JSON line with
+the keys the measurement contract asks for (metric, value, roofline,
+cpu_baseline, e2e with both copy directions, clocks, launch count), every
+leg of the run completing."""
+import json
+import os
+import subprocess
+import sys
+
+import pytest
+
+pytestmark = pytest.mark.gpu
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def test_bench_line_on_the_single_block_workload(cuda_ok, tmp_path):
+    out = tmp_path / "line.json"
+    cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--config", "c1", "--steps", "4", "--warmup", "3",
+           "--no-dit", "--cpu-budget-s", "2", "--out", str(out)]
+    res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+    assert res.returncode == 0, res.stderr[-2000:]
+    lines = [ln for ln in res.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1, res.stdout[-2000:]
+    line = json.loads(lines[0])
+    assert line == json.loads(out.read_text())
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step", "higher_is_better",
+              "scaling", "vs_baseline", "dtype", "data", "config", "roofline", "cpu_baseline", "e2e",
+              "e2e_unpadded", "clocks", "gpu_launches", "q_delta_roofline", "ms_per_step_serial",
+              "always_refresh_ms_per_step"):
+        assert k in line, k
+    assert line["value"] > 0 and line["steps"] == 4 and line["warmup"] == 3 and line["n_gpus"] == 1
+    assert line["higher_is_better"] is False and line["config"]["name"] == "c1"
+    assert line["gpu_launches"] > 0 and line["roofline"]["achieved"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] > 0
+    e2e = line["e2e"]
+    assert e2e["value"] > 0 and e2e["h2d_bytes_per_step"] > 0 and e2e["d2h_bytes_per_step"] > 0, e2e
+    assert line["e2e_unpadded"]["value"] > 0
