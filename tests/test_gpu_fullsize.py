@@ -182,34 +182,35 @@ def test_fullsize_depth_reduced_trajectory(cuda_ok):
             assert gm == [0] * len(blocks)
 
 
-def test_fullsize_trajectory_on_oracle_mass(cuda_ok):
-    """Image-edit workload, depth-reduced stack {0, 1, 44, 45, 59}, all 8
-    steps, D and M over the sampled target rows 0, 16, 32, ... (256 of 4096):
-    at every (t, b) the oracle computes M (Eq. 4) for all 24 heads from the
-    keys the block executed (the reference keys of its last materialisation,
-    kept by the oracle's own bookkeeping of Eq. 11) and D (Eq. 1) on the same
-    rows; the GPU's M must agree within 2e-5 and its D within the Q-change
-    tolerance, and the oracle's controller, fed with the oracle's own D and M
-    only, must reproduce every decision."""
+@pytest.mark.parametrize("name,blocks,k", [("c2", [0, 1, 44, 45, 59], 16), ("c3", [0, 1, 20, 39], 64)],
+                         ids=["image-edit", "video"])
+def test_fullsize_trajectory_on_oracle_mass(cuda_ok, name, blocks, k):
+    """Depth-reduced stacks of the image-edit (all 8 steps) and video (all 4
+    steps, per-head target-to-reference bias) workloads, D and M over the
+    sampled target rows 0, k, 2k, ... (256 rows): at every (t, b) the oracle
+    computes M (Eq. 4) for all 24 heads from the keys the block executed (the
+    reference keys of its last materialisation, kept by the oracle's own
+    bookkeeping of Eq. 11) and D (Eq. 1) on the same rows; the GPU's M must
+    agree within 2e-5 and its D within the Q-change tolerance, and the
+    oracle's controller, fed with the oracle's own D and M only, must
+    reproduce every decision."""
     from paper_2609_32415_gb300 import synth
-    k = 16
-    wl = synth.make_workload("c2")
-    blocks = [0, 1, 44, 45, 59]
+    wl = synth.make_workload(name)
     sub, rec = _run_stack(wl, blocks, sample_stride=k)
     sc = 1.0 / math.sqrt(sub.d)
+    bias = None if sub.bias is None else np.asarray(sub.bias)
     r0, r1 = sub.n_text, sub.n_text + sub.n_ref
     nb = len(blocks)
     gate = oracle.Gate(1, sub.theta, sub.delta_max, sub.forced_boundary)
     a_b = [-1] * nb                      # the oracle's own materialisation step per block
     m_prev = [None] * nb                 # the oracle's M of the previous step per block
     m_prev_gate = [None] * nb
-    m_err = 0.0
     for t in range(sub.n_steps):
         gate.begin_step(t)
         gm = [int(rec[(t, b)]["mode"][0]) for b in range(nb)]
         for b in range(nb):
             r = rec[(t, b)]
-            qt = _wide(_role(r["X"], sub, "tgt", 0)[0, :, ::k])            # [H, 256, d]
+            qt = _wide(_role(r["X"], sub, "tgt", 0)[0, :, ::k])            # [H, n_tgt / k, d]
             if t >= 1:
                 qp = _wide(_role(r["Xprev"], sub, "tgt", 0)[0, :, ::k])
                 D = oracle.q_change(qt, qp, sub.eps)                       # [H]
@@ -227,13 +228,13 @@ def test_fullsize_trajectory_on_oracle_mass(cuda_ok):
                                    _wide(_role(r["X"], sub, "tgt", 1)[0])], axis=1)
             vals = np.concatenate([_wide(_role(r["X"], sub, "text", 2)[0]), _wide(_role(Xk, sub, "ref", 2)[0]),
                                    _wide(_role(r["X"], sub, "tgt", 2)[0])], axis=1)
-            _, rm = oracle.joint_attention(qt, keys, vals, sc, ref_range=(r0, r1), want_o=False)
+            rb = np.ones(qt.shape[1], dtype=np.uint8) if bias is not None else None
+            _, rm = oracle.joint_attention(qt, keys, vals, sc, bias, rb, (r0, r1), want_o=False)
             M = oracle.exposure(rm)                                         # [H]
             # the GPU's M of this step's attention: its mass partials over the
             # sampled rows (text tiles hold zero), as the next step's gate sums them
             got = r["mass"][0].double().sum(-1).cpu().numpy() / qt.shape[1]
             err = np.abs(got - M).max()
-            m_err = max(m_err, err)
             assert err <= 2e-5, (t, b, err)
             m_prev[b] = M
             if t >= 1:   # the gate of step t read M of step t - 1 (its m_out)
