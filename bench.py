@@ -79,8 +79,23 @@ def parse_args():
                     help="skip the DiT-block stack summary that the default run adds to its line")
     ap.add_argument("--blocks", type=int, default=0,
                     help="run only the first N blocks of the stack (small profiling cases)")
+    ap.add_argument("--separate-cache-update", action="store_true",
+                    help="refresh each materialising block's cache slot with its own refadapt_ref_cache_update "
+                         "launch before the attention instead of inside it")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file")
-    return ap.parse_args()
+    args = ap.parse_args()
+    EXEC_OPTS["fused_cache"] = not args.separate_cache_update
+    return args
+
+
+# Executor options every timed schedule shares (set from the command line).
+EXEC_OPTS = {"fused_cache": True}
+
+
+def launches_per_block(t):
+    """Kernels one block of step t launches: Q change (t >= 1), gate,
+    attention, and the cache update unless it is fused into the attention."""
+    return (1 if t >= 1 else 0) + 2 + (0 if EXEC_OPTS["fused_cache"] else 1)
 
 
 # ----------------------------------------------------------------------------- helpers
@@ -303,7 +318,7 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
     ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, th, dm, wl.eps,
                   mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias,
                   log_steps=wl.n_steps, cue=cue, diagnostics=diagnostics, diag_row_stride=diag_row_stride,
-                  overlap=overlap)
+                  overlap=overlap, **EXEC_OPTS)
     views = [[roles_from_joint(inputs[t][b], wl.offsets(), wl.n) for b in range(wl.n_blocks)]
              for t in range(wl.n_steps)]
     T = wl.n_steps
@@ -336,7 +351,7 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
     for k in range(steps):
         t = (warmup + k) % T
         ex.step(t, views[t])
-        launches += wl.n_blocks * (4 if t >= 1 else 3)
+        launches += wl.n_blocks * launches_per_block(t)
         step_ev[k + 1].record()
     torch.cuda.synchronize()
     wall = time.perf_counter() - t0
@@ -377,7 +392,8 @@ def time_graphs(wl, inputs, warmup, steps):
     from paper_2609_32415_gb300 import Executor, roles_from_joint
     T = wl.n_steps
     ex = Executor(wl.n_blocks, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max, wl.eps,
-                  mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T)
+                  mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T,
+                  **EXEC_OPTS)
     views = [[roles_from_joint(inputs[t][b], wl.offsets(), wl.n) for b in range(wl.n_blocks)] for t in range(T)]
     for t in range(T):                            # eager pass: first-call set-up of every entry point
         ex.step(t, views[t])
@@ -453,12 +469,12 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
     previous-step mass partials and the controller state of the blocks before
     it); one device->host read of the step's modes (and gbar) follows; then,
     per block, the text Q/K/V and target K/V are copied, plus the reference
-    Q/K/V only when a sample materialises (a reusing block reads its reference
-    K/V from the cache), on a copy stream, triple-buffered and overlapped with
+    Q/K/V only when a sample materialises (COMPUTE or FULL; a reusing or
+    boundary block reads its reference Q/K/V from the cache), on a copy stream, triple-buffered and overlapped with
     the attentions (Executor.attend_block), up to two blocks ahead;
     consecutive attentions alternate between two high-priority streams; every
     executed row of the block's attention output (text and target rows, and
-    reference rows where a sample materialised) goes back to the host on a
+    reference rows where a sample is not REUSE) goes back to the host on a
     second copy stream as soon as the attention ends. A step ends when its
     last output is on the host.
 
@@ -532,7 +548,8 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
     NOUT = 3
     osl = [{r: torch.empty(shape[r], dtype=torch.bfloat16, device=dev) for r in ROLES} for _ in range(NOUT)]
     ex = Executor(nb, wl.B, wl.H, wl.d, wl.n_text, wl.n_ref, wl.n_tgt, wl.theta, wl.delta_max, wl.eps,
-                  mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T)
+                  mass_rows=wl.mass_rows, forced_boundary=wl.forced_boundary, bias=wl.bias, log_steps=T,
+                  **EXEC_OPTS)
     comp = torch.cuda.current_stream()
     copy = torch.cuda.Stream()
     back = torch.cuda.Stream()  # device -> host results
@@ -594,7 +611,10 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
         for st in attn_streams:
             st.wait_event(gates_done)
         decided.synchronize()
-        need_ref = [bool((modes_host[b] != 0).any()) for b in range(nb)]
+        # reference rows are read only by materialising samples (COMPUTE,
+        # FULL); they run (and come back) for every sample that is not REUSE
+        ref_in = [bool(((modes_host[b] == 2) | (modes_host[b] == 3)).any()) for b in range(nb)]
+        ref_out = [bool((modes_host[b] != 0).any()) for b in range(nb)]
         copy.wait_event(tq_free[1 - p])  # the next step's queries go where the previous step's were
         for b in range(nb):
             s = counter[0] % NSLOT
@@ -603,7 +623,7 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
             if b >= PREFETCH:
                 copy_base(t, b, s)
             with torch.cuda.stream(copy):
-                if need_ref[b]:
+                if ref_in[b]:
                     slots[s][size["base"]:].copy_(host[t][b]["ref"], non_blocking=True)
                     h2d[0] += size["ref"] * 2
                 ready = torch.cuda.Event()
@@ -623,7 +643,7 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
                 done.record(st)
             back.wait_event(done)
             with torch.cuda.stream(back):
-                for r in (("text", "ref", "tgt") if need_ref[b] else ("text", "tgt")):
+                for r in (("text", "ref", "tgt") if ref_out[b] else ("text", "tgt")):
                     hout[b][r].copy_(osl[o][r], non_blocking=True)
                     d2h[0] += osl[o][r].numel() * 2
                 out_free[o].record(back)
@@ -667,8 +687,8 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
     del host, slots, slot_v, osl, tq, ex, bufs, hout, arena
     pipeline = ("per step: the step's gates first (every block's target Q copied during the previous step), one "
                 "read of the modes, then per block text Q/K/V + target K/V and reference Q/K/V only where a "
-                "sample materialises, plus the next step's target Q; every executed output row (text and target, "
-                "reference where a sample materialised) back to the host behind each attention; bytes are the "
+                "sample materialises (COMPUTE or FULL), plus the next step's target Q; every executed output row "
+                "(text and target, reference where a sample is not REUSE) back to the host behind each attention; bytes are the "
                 "mean over the timed steps")
     return {"value": ms, "unit": "ms/step", "per_step_ms": per_step, "h2d_bytes_per_step": h2d_b,
             "d2h_bytes_per_step": d2h_b,

@@ -123,6 +123,30 @@ typedef struct {
  *                   when mass_rows = 1); the partials then sum the sampled
  *                   rows only (divide by their count). O is unaffected.
  *  err_word         device int32 or NULL; bit 0 set on a device timeout.
+ *
+ * Fused reference-cache update (paper Eq. 11; Algorithm 1's compute and full
+ * branches), optional: off when ref_fresh_q/k/v.ptr and a_b are all NULL
+ * (the zero-initialised struct). Otherwise, for
+ * every sample whose mode is RA_MODE_COMPUTE or RA_MODE_FULL, the reference
+ * K/V (and the reference query) are read from ref_fresh_k / ref_fresh_v /
+ * ref_fresh_q (this step's reference projections) instead of k/v/q[RA_REF],
+ * and copied into k/v/q[RA_REF] (the block's cache slot) as a by-product:
+ * the first CTA of each (sample, head) bulk-stores every reference K/V tile
+ * it streams through shared memory for its MMAs, each reference-row CTA its
+ * own query tiles, and a_b[b] = step. Samples in REUSE or BOUNDARY read the
+ * cache slot as before and leave it untouched. This replaces a separate
+ * refadapt_ref_cache_update (and its reads of the fresh tensors) on the
+ * attention's own pass over them.
+ *  ref_fresh_k/v    segments with n = k[RA_REF].n (16-byte aligned as above;
+ *                   ptr NULL only when n = 0).
+ *  ref_fresh_q      n = q[RA_REF].n when q[RA_REF] is given; ptr NULL and
+ *                   n = 0 otherwise.
+ *  a_b              device [B] int32 or NULL: materialisation step per sample.
+ *  step             the step index written into a_b.
+ * A fresh segment whose ptr equals its cache segment's (same strides) is read
+ * in place and not copied; K and V are both in place or both copied. The
+ * cache segments must not overlap the fresh ones otherwise. Errors
+ * (RA_EINVAL, nothing queued): n or stride mismatches as above.
  */
 typedef struct {
   int32_t B, H, d;
@@ -134,6 +158,10 @@ typedef struct {
   const int32_t* mode;
   float* mass_partial;
   int32_t* err_word;
+  ra_seg ref_fresh_q, ref_fresh_k, ref_fresh_v;  /* fused cache update; ref_fresh_k.ptr NULL = off */
+  int32_t* a_b;
+  int32_t step;
+  int32_t reserved;  /* set to 0 */
 } ra_attn_args;
 
 ra_status refadapt_joint_attn(const ra_attn_args* args, void* stream);

@@ -38,7 +38,8 @@ class RaAttnArgs(ctypes.Structure):
                 ("q", RaSeg * 3), ("k", RaSeg * 3), ("v", RaSeg * 3), ("o", RaSeg * 3),
                 ("softmax_scale", c_float), ("mass_row_stride", c_int32),
                 ("ref_logit_bias", c_void_p), ("mode", c_void_p), ("mass_partial", c_void_p),
-                ("err_word", c_void_p)]
+                ("err_word", c_void_p), ("ref_fresh_q", RaSeg), ("ref_fresh_k", RaSeg), ("ref_fresh_v", RaSeg),
+                ("a_b", c_void_p), ("step", c_int32), ("reserved", c_int32)]
 
 
 class RaGateArgs(ctypes.Structure):

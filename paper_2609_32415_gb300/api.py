@@ -51,8 +51,11 @@ def alloc_mass_partial(B, H, n_text, n_tgt, device="cuda"):
 
 
 def refadapt_joint_attn(q, k, v, o, mass_partial, mode=None, softmax_scale=0.0, ref_logit_bias=None,
-                        mass_rows=0, err_word=None, mass_row_stride=0, stream=None):
-    """q, k, v, o: sequences (text, ref, tgt) of [B, H, n, d] tensors; q[1] / o[1] may be None."""
+                        mass_rows=0, err_word=None, mass_row_stride=0, ref_fresh=None, a_b=None, step=0,
+                        stream=None):
+    """q, k, v, o: sequences (text, ref, tgt) of [B, H, n, d] tensors; q[1] / o[1] may be None.
+    ref_fresh: optional (q, k, v) of this step's reference rows for the fused
+    cache update (q may be None when q[1] is); a_b, step: the stamp it writes."""
     lib = _lib.load()
     B, H, _, d = k[2].shape
     a = RaAttnArgs()
@@ -69,6 +72,15 @@ def refadapt_joint_attn(q, k, v, o, mass_partial, mode=None, softmax_scale=0.0, 
     a.mode = _ptr(mode)
     a.mass_partial = _ptr(mass_partial)
     a.err_word = _ptr(err_word)
+    if ref_fresh is not None:
+        fq, fk, fv = ref_fresh
+        a.ref_fresh_q = seg(fq)
+        a.ref_fresh_k = seg(fk)
+        a.ref_fresh_v = seg(fv)
+        a.a_b = _ptr(a_b)
+        a.step = int(step)
+    elif a_b is not None:
+        raise ValueError("refadapt_joint_attn: a_b is written only with ref_fresh")
     return check("refadapt_joint_attn", lib.refadapt_joint_attn(ctypes.byref(a), _stream(stream)))
 
 

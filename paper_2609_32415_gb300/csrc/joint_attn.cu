@@ -27,9 +27,17 @@
 //               and the reference-only row sum l_ref (paper Eq. 4's inner sum
 //               is l_ref / l); then O / l -> bf16 global and the tile's sum of
 //               l_ref / l over its mass rows -> mass_partial.
+// Fused reference-cache update (paper Eq. 11), when the caller passes this
+// step's reference projections: samples in COMPUTE or FULL read reference
+// Q/K/V from them, and the producer thread copies what it streams into the
+// cache slot with TMA bulk-tensor stores from the swizzled stage buffers. The
+// first CTA of each (sample, head) stores every reference K/V tile one tile
+// after its load (the stage is refilled only once the store has read it);
+// each reference-row CTA stores its two Q tiles. Each byte of the fresh
+// reference rows is read from HBM once for both the MMAs and the copy.
 // Segment tails: TMA zero-fills rows past a segment's end; tail key tiles mask
 // the padded columns to -inf (probability 0) and the epilogue skips padded
-// query rows. Every mbarrier wait is bounded (WaitCtl); on a timeout the CTA
+// query rows; TMA stores clip rows past a segment's end. Every mbarrier wait is bounded (WaitCtl); on a timeout the CTA
 // drains its own TMA and MMA work, frees TMEM, flags the caller's error word
 // and returns.
 #include <cuda.h>
@@ -77,6 +85,7 @@ struct Params {
   CUtensorMap tm_q[3];
   CUtensorMap tm_k[3];
   CUtensorMap tm_v[3];
+  CUtensorMap tm_qf, tm_kf, tm_vf;  // this step's reference rows (fused cache update)
   __nv_bfloat16* o_ptr[3];
   int64_t o_sb[3], o_sh[3], o_sn[3];
   int32_t nq[3];  // query rows per role
@@ -93,8 +102,30 @@ struct Params {
   const int32_t* mode;
   float* mass_partial;
   int32_t* err_word;
+  int32_t* a_b;
+  int32_t step;
+  int32_t fresh;     // refreshing samples read reference rows from tm_*f
+  int32_t store_kv;  // ... and copy those K / V tiles into tm_k[1] / tm_v[1]
+  int32_t store_q;   // ... and those Q tiles into tm_q[1]
   uint64_t budget_ns;
 };
+
+__device__ __forceinline__ bool refreshes(int m) { return m == RA_MODE_COMPUTE || m == RA_MODE_FULL; }
+
+// Tile (c0 = column, c1 = row, c2 = head, c3 = sample) of a 4-D tensor map,
+// shared -> global, bulk-group completion; rows past the tensor are clipped.
+__device__ __forceinline__ void tma_store_4d(const void* tmap, const void* src, int32_t c0, int32_t c1,
+                                             int32_t c2, int32_t c3) {
+  asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%2, %3, %4, %5}], [%1];" ::"l"(
+                   reinterpret_cast<uint64_t>(tmap)),
+               "r"(smem_u32(src)), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+               : "memory");
+}
+__device__ __forceinline__ void bulk_commit() { asm volatile("cp.async.bulk.commit_group;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_read_all() { asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory"); }
+__device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Shared memory written by TMA loads (async proxy) is next read by TMA stores.
+__device__ __forceinline__ void fence_proxy_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 
 __device__ __forceinline__ void kv_tile(const Params& p, int j, int& r, int& row0) {
   if (j < p.kv_tiles[0]) {
@@ -245,17 +276,52 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
     if (warp == 0) {
       if (lane == 0) {
         // ------------------------------------------------------------ TMA producer
-        tma_prefetch_desc(&p.tm_q[role]);
+        const bool fresh = p.fresh && refreshes(mode);
+        const bool store_kv = fresh && p.store_kv && blockIdx.x == 0;
+        const bool store_q = fresh && p.store_q && role == 1;
+        const CUtensorMap* tq = (role == 1 && fresh) ? &p.tm_qf : &p.tm_q[role];
+        if (fresh && blockIdx.x == 0 && h == 0 && p.a_b) p.a_b[b] = p.step;
+        tma_prefetch_desc(tq);
         for (int r = 0; r < 3; ++r)
           if (p.kv_tiles[r] > 0) {
-            tma_prefetch_desc(&p.tm_k[r]);
-            tma_prefetch_desc(&p.tm_v[r]);
+            tma_prefetch_desc((r == 1 && fresh) ? &p.tm_kf : &p.tm_k[r]);
+            tma_prefetch_desc((r == 1 && fresh) ? &p.tm_vf : &p.tm_v[r]);
           }
         int k_issued = 0, v_issued = 0;  // K / V tiles whose loads were issued
+        uint32_t stored_stages = 0;      // stages whose last tile has a store that may still read it
+        bool q_stored = !store_q;
+        // Copy tile jj (loaded by now or soon) into the cache slot if it is a
+        // reference tile; the Q tiles go with the first call.
+        auto store_tiles = [&](int jj) -> bool {
+          if (!q_stored) {
+            if (!mbar_wait(q_full, 0, ctl)) return false;
+            fence_proxy_async_smem();
+            for (int t = 0; t < (has_b ? 2 : 1); ++t)
+              for (int c = 0; c < C::CHUNKS; ++c)
+                tma_store_4d(&p.tm_q[1], smem + C::OFF_Q + t * C::TILE_BYTES + c * C::CHUNK_BYTES, c * 64,
+                             (tileA + t) * BM, h, b);
+            bulk_commit();
+            q_stored = true;
+          }
+          int r, row0;
+          kv_tile(p, jj, r, row0);
+          if (!store_kv || r != 1) return true;
+          const int s = jj % S;
+          const uint32_t ph = (jj / S) & 1;
+          if (!mbar_wait(k_full + s, ph, ctl) || !mbar_wait(v_full + s, ph, ctl)) return false;
+          fence_proxy_async_smem();
+          for (int c = 0; c < C::CHUNKS; ++c) {
+            tma_store_4d(&p.tm_k[1], smem + C::OFF_K + s * C::TILE_BYTES + c * C::CHUNK_BYTES, c * 64, row0, h, b);
+            tma_store_4d(&p.tm_v[1], smem + C::OFF_V + s * C::TILE_BYTES + c * C::CHUNK_BYTES, c * 64, row0, h, b);
+          }
+          bulk_commit();
+          stored_stages |= 1u << s;
+          return true;
+        };
         mbar_arrive_expect_tx(q_full, C::TILE_BYTES * (has_b ? 2 : 1));
         for (int t = 0; t < (has_b ? 2 : 1); ++t)
           for (int c = 0; c < C::CHUNKS; ++c)
-            tma_load_4d(smem + C::OFF_Q + t * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_q[role], q_full, c * 64,
+            tma_load_4d(smem + C::OFF_Q + t * C::TILE_BYTES + c * C::CHUNK_BYTES, tq, q_full, c * 64,
                         (tileA + t) * BM, h, b);
         for (int j = 0; j < nkv; ++j) {
           const int s = j % S;
@@ -263,18 +329,27 @@ __global__ void __launch_bounds__(NUM_THREADS, 1) joint_attn_kernel(const __grid
           int r, row0;
           kv_tile(p, j, r, row0);
           if (j >= S && !mbar_wait(k_empty + s, ph ^ 1, ctl)) break;
+          if (stored_stages & (1u << s)) {  // stage s still feeds a store of tile j - S
+            bulk_wait_read_all();
+            stored_stages = 0;
+          }
           mbar_arrive_expect_tx(k_full + s, C::TILE_BYTES);
           for (int c = 0; c < C::CHUNKS; ++c)
-            tma_load_4d(smem + C::OFF_K + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_k[r], k_full + s,
-                        c * 64, row0, h, b);
+            tma_load_4d(smem + C::OFF_K + s * C::TILE_BYTES + c * C::CHUNK_BYTES,
+                        (r == 1 && fresh) ? &p.tm_kf : &p.tm_k[r], k_full + s, c * 64, row0, h, b);
           ++k_issued;
           if (j >= S && !mbar_wait(v_empty + s, ph ^ 1, ctl)) break;
           mbar_arrive_expect_tx(v_full + s, C::TILE_BYTES);
           for (int c = 0; c < C::CHUNKS; ++c)
-            tma_load_4d(smem + C::OFF_V + s * C::TILE_BYTES + c * C::CHUNK_BYTES, &p.tm_v[r], v_full + s,
-                        c * 64, row0, h, b);
+            tma_load_4d(smem + C::OFF_V + s * C::TILE_BYTES + c * C::CHUNK_BYTES,
+                        (r == 1 && fresh) ? &p.tm_vf : &p.tm_v[r], v_full + s, c * 64, row0, h, b);
           ++v_issued;
+          if (j >= 1 && (store_kv || store_q) && !store_tiles(j - 1)) break;
         }
+        if ((store_kv || store_q) && !*abort_flag && v_issued == nkv) store_tiles(nkv - 1);
+        // Shared memory must outlive the reads of every store issued; the
+        // cache slot is complete when the kernel is.
+        if (store_kv || store_q) bulk_wait_all();
         if (*abort_flag) {
           // Let every load this thread issued land before the CTA exits: stage s
           // received loads for j = s, s + S, ...; wait for the last one's phase.
@@ -582,6 +657,60 @@ extern "C" ra_status refadapt_joint_attn(const ra_attn_args* a, void* stream) {
     p.o_sb[r] = a->o[r].stride_b;
     p.o_sh[r] = a->o[r].stride_h;
     p.o_sn[r] = a->o[r].stride_n;
+  }
+  if (a->ref_fresh_q.ptr != nullptr || a->ref_fresh_k.ptr != nullptr || a->ref_fresh_v.ptr != nullptr ||
+      a->a_b != nullptr) {
+    // Fused cache update: this step's reference rows, read by refreshing
+    // samples and copied into the segments k/v/q[RA_REF] point at.
+    const ra_seg* fr[3] = {&a->ref_fresh_q, &a->ref_fresh_k, &a->ref_fresh_v};
+    const ra_seg* ca[3] = {&a->q[RA_REF], &a->k[RA_REF], &a->v[RA_REF]};
+    const char* kinds[3] = {"q", "k", "v"};
+    bool copy[3] = {false, false, false};
+    for (int i = 0; i < 3; ++i) {
+      if (i == 0 && !ref_rows) {
+        if (fr[0]->ptr != nullptr || fr[0]->n != 0) {
+          set_error("refadapt_joint_attn: ref_fresh_q given without reference query rows (q[ref] is NULL)");
+          return RA_EINVAL;
+        }
+        continue;
+      }
+      snprintf(what, sizeof(what), "refadapt_joint_attn: ref_fresh_%s", kinds[i]);
+      if (!check_seg(*fr[i], what)) return RA_EINVAL;
+      if (fr[i]->n != ca[i]->n) {
+        set_error("refadapt_joint_attn: ref_fresh_%s has n = %d, %s[ref] has %d", kinds[i], fr[i]->n, kinds[i],
+                  ca[i]->n);
+        return RA_EINVAL;
+      }
+      if (fr[i]->ptr == ca[i]->ptr) {
+        if (fr[i]->stride_b != ca[i]->stride_b || fr[i]->stride_h != ca[i]->stride_h ||
+            fr[i]->stride_n != ca[i]->stride_n) {
+          set_error("refadapt_joint_attn: ref_fresh_%s shares its pointer with %s[ref] but not its strides",
+                    kinds[i], kinds[i]);
+          return RA_EINVAL;
+        }
+        continue;  // read in place
+      }
+      copy[i] = true;
+      if (fr[i]->n > 0) {
+        CUtensorMap* tm = (i == 0) ? &p.tm_qf : (i == 1) ? &p.tm_kf : &p.tm_vf;
+        if (!encode_seg(tm, *fr[i], a->B, a->H, d, 64, (i == 0) ? BM : BN, true)) return RA_EINVAL;
+      }
+    }
+    if (copy[1] != copy[2]) {
+      set_error("refadapt_joint_attn: ref_fresh_k and ref_fresh_v must both be in place or both be copied");
+      return RA_EINVAL;
+    }
+    // Segments read in place keep their own maps as the fresh ones.
+    if (!copy[0]) p.tm_qf = p.tm_q[RA_REF];
+    if (!copy[1]) {
+      p.tm_kf = p.tm_k[RA_REF];
+      p.tm_vf = p.tm_v[RA_REF];
+    }
+    p.fresh = 1;
+    p.store_kv = copy[1] ? 1 : 0;
+    p.store_q = copy[0] ? 1 : 0;
+    p.a_b = a->a_b;
+    p.step = a->step;
   }
   p.B = a->B;
   p.H = a->H;

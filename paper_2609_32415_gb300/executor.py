@@ -8,9 +8,11 @@ Executor.step); overlap=False keeps every launch on the caller's stream.
 Per block b the executor owns the cache state of paper Eq. 11: reference K and
 V, the cached reference hidden state (here the reference query, which is what
 restoring the hidden state at a boundary produces in this hot path) and a_b.
-The joint-attention kernel always reads reference Q/K/V from that cache slot:
-COMPUTE / FULL blocks refresh the slot first (so they see fresh values),
-REUSE and BOUNDARY blocks see the values of the last materialisation.
+REUSE and BOUNDARY blocks read reference Q/K/V from that cache slot (the
+values of the last materialisation). COMPUTE / FULL blocks read this step's
+reference rows, and the joint-attention kernel copies them into the slot in
+the same pass (fused_cache, the default); fused_cache=False refreshes the slot
+with refadapt_ref_cache_update first and the attention reads the slot.
 """
 import torch
 
@@ -63,12 +65,16 @@ class Executor:
     stream for the decisions and cache updates, two higher-priority streams
     for the attentions), forked from and joined to the caller's stream per
     step; the results equal the one-stream order bit for bit.
+
+    ``fused_cache`` (default) lets the attention of a materialising block
+    write its cache slot (refadapt_joint_attn's ref_fresh arguments) instead
+    of a refadapt_ref_cache_update launch before it; the results are the same.
     """
 
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
                  mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
                  device="cuda", cue="product", diagnostics=False, diag_row_stride=1, sample_stride=1,
-                 overlap=True):
+                 overlap=True, fused_cache=True):
         if cue not in CUES:
             raise ValueError("unknown cue %r" % (cue,))
         self.cue = cue
@@ -99,6 +105,7 @@ class Executor:
         # update on a side stream one block ahead, in the previous attention's
         # tail wave (SMs its last wave leaves idle); see step().
         self.overlap = bool(overlap)
+        self.fused_cache = bool(fused_cache)
         if self.overlap:
             # The attentions run on a high-priority stream and the side work on
             # a default-priority one: the CTA scheduler serves pending attention
@@ -185,8 +192,9 @@ class Executor:
         """The attention half of block b of step t, after gate_block(t, b): the
         reference cache update (materialising samples) and the joint attention
         with the mass partials. x[ref] is read only for samples whose mode is
-        not REUSE."""
-        self.update_cache(t, b, x, log_index, stream)
+        COMPUTE or FULL."""
+        if not self.fused_cache:
+            self.update_cache(t, b, x, log_index, stream)
         self.attend(t, b, x, out, log_index, stream)
 
     def update_cache(self, t, b, x, log_index=None, stream=None):
@@ -199,8 +207,10 @@ class Executor:
                                       x_src=qr, x_cache=self.cache_x[b], stream=stream)
 
     def attend(self, t, b, x, out, log_index=None, stream=None):
-        """Block b's joint attention of step t (after its gate and cache
-        update), with the mass partials the next step's gate reads."""
+        """Block b's joint attention of step t (after its gate, and after its
+        cache update unless fused_cache), with the mass partials the next
+        step's gate reads. With fused_cache, materialising samples read x[ref]
+        and the kernel writes it into the cache slot and stamps a_b = t."""
         li = (t % self.log_steps) if log_index is None else log_index
         mode = self.modes[li, b]
         qt = x["tgt"][0]
@@ -212,7 +222,9 @@ class Executor:
             (x["text"][2], self.cache_v[b], x["tgt"][2]),
             (out["text"], out["ref"], out["tgt"]),
             self.mass[b], mode=mode, softmax_scale=self.softmax_scale, ref_logit_bias=self.bias,
-            mass_rows=self.mass_rows, err_word=self.err, mass_row_stride=self.sample_stride, stream=stream)
+            mass_rows=self.mass_rows, err_word=self.err, mass_row_stride=self.sample_stride,
+            ref_fresh=x["ref"] if self.fused_cache else None,
+            a_b=self.a_b[b] if self.fused_cache else None, step=t, stream=stream)
         if self.attn_hook is not None:
             self.attn_hook("post", t, b)
         if self.diagnostics:
@@ -270,7 +282,8 @@ class Executor:
                 side.wait_event(self._attn_done[b - 2])
             with torch.cuda.stream(side):
                 self.gate_block(t, b, inputs[b]["tgt"][0], log_index)
-                self.update_cache(t, b, inputs[b], log_index)
+                if not self.fused_cache:
+                    self.update_cache(t, b, inputs[b], log_index)
                 self._decided[b].record(side)
             with torch.cuda.stream(main):
                 main.wait_event(self._decided[b])

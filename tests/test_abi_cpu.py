@@ -49,6 +49,8 @@ int main(void) {
   printf("%zu %zu %zu\n", sizeof(ra_seg), sizeof(ra_attn_args), sizeof(ra_gate_args));
   printf("%zu %zu %zu %zu\n", offsetof(ra_attn_args, q), offsetof(ra_attn_args, softmax_scale),
          offsetof(ra_attn_args, mode), offsetof(ra_attn_args, err_word));
+  printf("%zu %zu %zu %zu\n", offsetof(ra_attn_args, ref_fresh_q), offsetof(ra_attn_args, ref_fresh_v),
+         offsetof(ra_attn_args, a_b), offsetof(ra_attn_args, step));
   printf("%zu %zu %zu\n", offsetof(ra_gate_args, t), offsetof(ra_gate_args, q_delta),
          offsetof(ra_gate_args, m_out));
   return 0;
@@ -61,7 +63,8 @@ int main(void) {
     got = [int(x) for x in out]
     want = [ctypes.sizeof(RaSeg), ctypes.sizeof(RaAttnArgs), ctypes.sizeof(RaGateArgs),
             RaAttnArgs.q.offset, RaAttnArgs.softmax_scale.offset, RaAttnArgs.mode.offset,
-            RaAttnArgs.err_word.offset, RaGateArgs.t.offset, RaGateArgs.q_delta.offset,
+            RaAttnArgs.err_word.offset, RaAttnArgs.ref_fresh_q.offset, RaAttnArgs.ref_fresh_v.offset,
+            RaAttnArgs.a_b.offset, RaAttnArgs.step.offset, RaGateArgs.t.offset, RaGateArgs.q_delta.offset,
             RaGateArgs.m_out.offset]
     assert got == want
 

@@ -42,6 +42,7 @@ def _run_stack(wl, blocks, sample_stride=1):
                   bias=sub.bias, log_steps=sub.n_steps, sample_stride=sample_stride)
     rec = {}
     prev = {}
+    last = {}  # (block, sample) -> (inputs, step) of the last materialisation
     for t in range(sub.n_steps):
         for b in range(sub.n_blocks):
             X = traj.get(t, b)
@@ -49,6 +50,15 @@ def _run_stack(wl, blocks, sample_stride=1):
                                  device="cuda") for r in ROLES}
             ex.block(t, b, roles_from_joint(X, sub.offsets(), sub.n), out)
             torch.cuda.synchronize()
+            # Eq. 11: the cache slot holds the reference Q/K/V of the block's
+            # last materialisation, bit for bit, and a_b its step
+            for s, m in enumerate(ex.modes[t, b].tolist()):
+                if m in (2, 3):
+                    last[(b, s)] = (X, t)
+                src, ts = last[(b, s)]
+                for z, cache in enumerate((ex.cache_x, ex.cache_k, ex.cache_v)):
+                    assert torch.equal(cache[b][s], _role(src, sub, "ref", z)[s]), (t, b, s, z)
+                assert int(ex.a_b[b][s]) == ts, (t, b, s)
             rec[(t, b)] = {"X": X, "O": out, "D": ex.D[b].clone(), "mode": ex.modes[t, b].clone(),
                            "gbar": ex.gbar[t, b].clone(), "mass": ex.mass[b].clone(),
                            "M": ex.M[t, b].clone(), "Xprev": prev.get(b)}
