@@ -124,9 +124,12 @@ ATTN_SOURCES = ("paper_2609_32415_gb300/csrc/joint_attn.cu", "paper_2609_32415_g
 def recorded_traffic(config, modes=None):
     """DRAM bytes per attention launch from the committed ncu summary, or None
     when the kernel source changed since the counters were taken. A record with
-    separate refresh and reuse launches is averaged over the timed launches'
-    modes (`modes`: one list of per-sample modes per launch; a launch counts as
-    refresh when any sample materialises)."""
+    separate launch kinds is averaged over the timed launches' modes (`modes`:
+    one list of per-sample modes per launch). Kinds: "materialise" (a sample in
+    COMPUTE or FULL: all rows, and the kernel writes the cache slot),
+    "refresh" (a BOUNDARY sample: all rows, no cache write) and "reuse"; a
+    record without "materialise" counts every launch that runs reference rows
+    as "refresh"."""
     path = os.path.join(ROOT, "profiles", "attn_traffic.json")
     try:
         with open(path) as f:
@@ -140,11 +143,18 @@ def recorded_traffic(config, modes=None):
         return r
     if not modes or "refresh" not in r or "reuse" not in r:
         return None
-    n_ref = sum(1 for m in modes if any(int(x) != 0 for x in m))
-    n_reu = len(modes) - n_ref
-    out = {"bytes": int(round((n_ref * r["refresh"]["bytes"] + n_reu * r["reuse"]["bytes"]) / len(modes))),
-           "mix": {"refresh_launches": n_ref, "reuse_launches": n_reu},
-           "refresh": r["refresh"], "reuse": r["reuse"], "capture": r.get("capture")}
+
+    def kind(m):
+        m = [int(x) for x in m]
+        if "materialise" in r and any(x in (2, 3) for x in m):
+            return "materialise"
+        return "refresh" if any(x != 0 for x in m) else "reuse"
+
+    kinds = [kind(m) for m in modes]
+    mix = {k: kinds.count(k) for k in ("materialise", "refresh", "reuse") if k in r}
+    out = {"bytes": int(round(sum(r[k]["bytes"] for k in kinds) / len(kinds))),
+           "mix": {k + "_launches": v for k, v in mix.items()}, "capture": r.get("capture")}
+    out.update({k: r[k] for k in mix})
     return out
 
 

@@ -138,10 +138,10 @@ class DiTExecutor:
              "k_norm": Ws["ref"]["k_norm"], "pos_offset": self.pos0["ref"], "gated": True}],
             3 * C, C, RA_EPI_QKV, mode=mode, rope=self.rope, H=self.H, d=self.d, norm_eps=self.norm_eps,
             err_word=self.err, stream=stream)
-        # a_b = t for COMPUTE / FULL samples (the K/V were written in place)
-        api.refadapt_ref_cache_update(self.cache_k[b], self.cache_v[b], self.cache_k[b], self.cache_v[b], mode, t,
-                                      self.a_b[b], stream=stream)
-        # 4. joint attention (mass partials of the executed attention)
+        # 4. joint attention (mass partials of the executed attention). The
+        # reference K/V were written into the cache slot in place, so the fresh
+        # reference rows are the slot itself: the kernel copies nothing and
+        # stamps a_b = t for COMPUTE / FULL samples.
         if self.attn_hook is not None:
             self.attn_hook("pre", t, b)
         api.refadapt_joint_attn(
@@ -149,7 +149,8 @@ class DiTExecutor:
             (self.qkv["text"][1], self.cache_k[b], self.qkv["tgt"][1]),
             (self.qkv["text"][2], self.cache_v[b], self.qkv["tgt"][2]),
             tuple(self._heads(self.o[r]) for r in ROLES),
-            self.mass[b], mode=mode, mass_rows=self.mass_rows, err_word=self.err, stream=stream)
+            self.mass[b], mode=mode, mass_rows=self.mass_rows, err_word=self.err,
+            ref_fresh=(self.q_ref, self.cache_k[b], self.cache_v[b]), a_b=self.a_b[b], step=t, stream=stream)
         if self.attn_hook is not None:
             self.attn_hook("post", t, b)
         # 5. output projection with the gated residual (reference: H_b -> h1_ref)

@@ -60,6 +60,11 @@ def _run(wl, di, theta, delta_max, forced_boundary=-1, cue="product"):
     modes = ex.modes.cpu().numpy()
     gbar = ex.gbar.double().cpu().numpy()
     M = ex.M.double().cpu().numpy()
+    # a_b (Eq. 11): the last step at which the block materialised, per sample
+    for b in range(wl.n_blocks):
+        for s in range(wl.B):
+            mat = [t for t in range(wl.n_steps) if modes[t, b, s] in (COMPUTE, FULL)]
+            assert int(ex.a_b[b, s]) == (mat[-1] if mat else -1), (b, s)
 
     def h_in(t):
         return {r: bits(x) for r, x in inputs[t].items()}
