@@ -759,7 +759,8 @@ def time_q_delta_long(n_tgt=16380, H=24, d=128, eps=1e-6, reps=64):
 
 def time_q_delta(wl, inputs, reps=64):
     """HBM roofline of the Q-change reduction alone: target Q of step 1 vs step
-    0, rotating over 8 blocks (8 x 50 MB > L2, so every launch reads HBM).
+    0, rotating over 8 blocks (8 x 50 MB > L2, so every launch reads HBM; a
+    stack cut to fewer blocks is padded with seeded pairs of the same shape).
     The launches are queued behind a GPU-side sleep so they run back to back;
     the average launch duration is the events' span divided by the launches."""
     import torch
@@ -767,6 +768,13 @@ def time_q_delta(wl, inputs, reps=64):
     nb = min(8, wl.n_blocks)
     pairs = [(roles_from_joint(inputs[1][b], wl.offsets(), wl.n)["tgt"][0],
               roles_from_joint(inputs[0][b], wl.offsets(), wl.n)["tgt"][0]) for b in range(nb)]
+    g = torch.Generator(device="cuda")
+    g.manual_seed(0x0DE17A)
+    shape = (wl.B, wl.H, wl.n_tgt, wl.d)
+    while len(pairs) < 8:
+        prev = (torch.randn(shape, generator=g, device="cuda") / wl.d ** 0.5).to(torch.bfloat16)
+        cur = (prev.float() + 0.3 * torch.randn(shape, generator=g, device="cuda") / wl.d ** 0.5).to(torch.bfloat16)
+        pairs.append((cur, prev))
     ms = _q_delta_launch_ms(pairs, wl.B, wl.H, wl.eps, reps)
     byts = 4 * wl.n_tgt * wl.H * wl.d * wl.B
     # Context: a library streaming read of the same number of bytes (torch's
