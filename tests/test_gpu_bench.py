@@ -36,3 +36,20 @@ def test_bench_line_on_the_single_block_workload(cuda_ok, tmp_path):
     e2e = line["e2e"]
     assert e2e["value"] > 0 and e2e["h2d_bytes_per_step"] > 0 and e2e["d2h_bytes_per_step"] > 0, e2e
     assert line["e2e_unpadded"]["value"] > 0
+
+
+def test_bench_separate_cache_update_schedule(cuda_ok):
+    """--separate-cache-update adds one refadapt_ref_cache_update launch per
+    block and step to the count; the same trajectory's modes either way."""
+    def line(extra):
+        cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--config", "c1", "--steps", "4", "--warmup", "3",
+               "--no-dit", "--no-e2e", "--no-cpu-baseline", "--no-refresh-baseline", "--no-graph", "--no-serial",
+               "--no-nested"] + extra
+        res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
+        assert res.returncode == 0, res.stderr[-2000:]
+        return json.loads([ln for ln in res.stdout.splitlines() if ln.startswith("{")][-1])
+
+    fused, separate = line([]), line(["--separate-cache-update"])
+    assert fused["modes_per_step"] == separate["modes_per_step"]
+    blocks = fused["config"]["blocks"]
+    assert separate["gpu_launches"] - fused["gpu_launches"] == blocks * fused["steps"]
