@@ -13,10 +13,11 @@ tests/test_oracle_pins.py and tests/test_oracle_dit_pins.py against brute
 force, closed forms, library special cases and invariants; none is "parity
 unpinned".
 """
-from .core import (REUSE, BOUNDARY, COMPUTE, FULL, ROLES, Gate, attention_flops,
+from .core import (REUSE, BOUNDARY, COMPUTE, FULL, ROLES, Gate, adjacent_ref_mass_change, attention_flops,
                    bf16_to_f64, block_attention, closed_loop, default_threads, endpoint_drift, exposure,
-                   joint_attention, local_impact, q_change, reuse_score_fraction)
+                   head_mean_exposure, joint_attention, local_impact, q_change, reuse_score_fraction)
 
-__all__ = ["REUSE", "BOUNDARY", "COMPUTE", "FULL", "ROLES", "Gate", "attention_flops",
-           "bf16_to_f64", "block_attention", "closed_loop", "default_threads", "endpoint_drift", "exposure",
-           "joint_attention", "local_impact", "q_change", "reuse_score_fraction"]
+__all__ = ["REUSE", "BOUNDARY", "COMPUTE", "FULL", "ROLES", "Gate", "adjacent_ref_mass_change",
+           "attention_flops", "bf16_to_f64", "block_attention", "closed_loop", "default_threads",
+           "endpoint_drift", "exposure", "head_mean_exposure", "joint_attention", "local_impact", "q_change",
+           "reuse_score_fraction"]

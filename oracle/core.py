@@ -11,6 +11,9 @@ Each function names the passage of the paper it restates:
                            the inner sum of Eq. 4 (C part in attn_oracle.c).
 * ``exposure``             Eq. 4: mean over target query rows of the softmax
                            mass on reference keys.
+* ``head_mean_exposure``   Eq. 5: the mean of Eq. 4 over heads.
+* ``adjacent_ref_mass_change``  Eq. 6: mean absolute change of Eq. 5 between
+                           neighbouring steps of a block, in percentage points.
 * ``q_change``             Eq. 1 applied to each post-RoPE target-query head
                            (Sec. 4, "Runtime cues observable under reuse").
 * ``Gate``                 Eq. 12 (per-head product), the head mean of App. A.2,
@@ -147,6 +150,29 @@ def exposure(row_mass_tgt, row_mass_text=None) -> np.ndarray:
         parts.append(np.asarray(row_mass_text, dtype=np.float64))
     allm = np.concatenate(parts, axis=1)
     return allm.sum(axis=1) / allm.shape[1]
+
+
+def head_mean_exposure(M) -> np.ndarray:
+    """Eq. 5: (1/H) sum_h M_{t,b,h}; M [..., H] -> [...]."""
+    M = np.asarray(M, dtype=np.float64)
+    total = np.zeros(M.shape[:-1])
+    for h in range(M.shape[-1]):
+        total = total + M[..., h]
+    return total / M.shape[-1]
+
+
+def adjacent_ref_mass_change(Mbar) -> np.ndarray:
+    """Eq. 6: (100 / (T - 1)) sum_{t=2}^{T} |Mbar_t - Mbar_{t-1}|, in
+    percentage points. Mbar [T, ...] holds the head-mean exposure of steps
+    1..T (first axis) of a block; T >= 2."""
+    Mbar = np.asarray(Mbar, dtype=np.float64)
+    T = Mbar.shape[0]
+    if T < 2:
+        raise ValueError("Eq. 6 needs at least two steps")
+    total = np.zeros(Mbar.shape[1:])
+    for t in range(1, T):
+        total = total + np.abs(Mbar[t] - Mbar[t - 1])
+    return 100.0 * total / (T - 1)
 
 
 def attention_flops(n_q, n_k, H, d) -> int:

@@ -309,5 +309,34 @@ class Executor:
             self.step(t, inputs, outs, log_index)
         return g
 
+    def exposure_summary(self, n_steps, fresh=False):
+        """The exposure summaries of Sec. 3.2 over the logged steps
+        0 .. n_steps - 1 of a trajectory (n_steps <= log_steps, read after the
+        steps have run): the head-mean exposure of Eq. 5, Mbar [n_steps,
+        blocks, B], and its mean adjacent-step change of Eq. 6 in percentage
+        points, Delta [blocks, B] (fp64 numpy arrays).
+
+        fresh=False takes the executed attention's exposure, the one the
+        controller reads: step t's is what step t + 1's gate logged, the last
+        step's comes from the current mass partials. fresh=True takes the
+        fresh-reference pass of the diagnostics (A^fresh, the paper's
+        summaries); it needs diagnostics=True. A summary of logged results
+        for analysis, read back to the host; no part of a step."""
+        import numpy as np
+        T = int(n_steps)
+        if T < 2 or T > self.log_steps:
+            raise ValueError("exposure_summary: need 2 <= n_steps <= log_steps (%d)" % self.log_steps)
+        if fresh:
+            if not self.diagnostics:
+                raise ValueError("exposure_summary(fresh=True) needs Executor(diagnostics=True)")
+            M = self.M_fresh_part[:T].double().sum(-1).cpu().numpy() / float(self.n_tgt_sampled)
+        else:
+            M = np.empty((T, self.n_blocks, self.B, self.H))
+            M[:T - 1] = self.M[1:T].double().cpu().numpy()
+            M[T - 1] = self.mass.double().sum(-1).cpu().numpy() / float(self.mass_row_count)
+        Mbar = M.mean(axis=-1)
+        Delta = 100.0 * np.abs(np.diff(Mbar, axis=0)).sum(axis=0) / (T - 1)
+        return Mbar, Delta
+
     def check(self, stream=None):
         api.refadapt_check_error(self.err, stream)

@@ -55,7 +55,9 @@ def _run_both(wl, o_sample=None, cue="product", diagnostics=False, diag_row_stri
         rows_s = ex.n_tgt_sampled
         diag = {"E_K": ex.E_K.double().cpu().numpy(), "E_V": ex.E_V.double().cpu().numpy(),
                 "I_KV": ex.I_KV.double().cpu().numpy(),
-                "M_fresh": ex.M_fresh_part.double().sum(-1).cpu().numpy() / rows_s}
+                "M_fresh": ex.M_fresh_part.double().sum(-1).cpu().numpy() / rows_s,
+                "summary": ex.exposure_summary(wl.n_steps),
+                "summary_fresh": ex.exposure_summary(wl.n_steps, fresh=True)}
         return modes, gbar, Mlog, D, outs, rec, diag
     return modes, gbar, Mlog, D, outs, rec
 
@@ -151,6 +153,16 @@ def test_closed_loop_staleness_diagnostics(cuda_ok):
                 assert ok.all(), (t, b, key, got, want)
             assert np.abs(diag["M_fresh"][t, b] - r["M_fresh"]).max() <= M_ABS, (t, b)
             assert np.abs(diag["I_KV"][t, b] - r["I_KV"]).max() <= 5e-3, (t, b, diag["I_KV"][t, b], r["I_KV"])
+    # Eqs. 5-6 over the trajectory, executed and fresh exposure, against the
+    # oracle's summaries of its own M (M within M_ABS, so Mbar within M_ABS
+    # and Delta within 2 * 100 * M_ABS percentage points)
+    for key, src in (("summary", "M"), ("summary_fresh", "M_fresh")):
+        Mo = np.stack([np.stack([rec[t][b][src] for b in range(wl.n_blocks)]) for t in range(wl.n_steps)])
+        Mbar_o = oracle.head_mean_exposure(Mo)
+        Delta_o = oracle.adjacent_ref_mass_change(Mbar_o)
+        Mbar, Delta = diag[key]
+        assert np.abs(Mbar - Mbar_o).max() <= M_ABS, key
+        assert np.abs(Delta - Delta_o).max() <= 200 * M_ABS, (key, Delta, Delta_o)
 
 
 def test_closed_loop_sampled_target_rows(cuda_ok):

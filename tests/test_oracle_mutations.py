@@ -60,6 +60,16 @@ MUTATIONS = [
      [(P, "test_q_change_brute_force", ())]),
     ("bf16_shift", "core.py", "<< np.uint32(16)", "<< np.uint32(15)",
      [(P, "test_bf16_widening_known_patterns", ())]),
+    # Eqs. 5-6, the exposure summaries (core.py)
+    ("eq5_drops_last_head", "core.py", "for h in range(M.shape[-1]):", "for h in range(M.shape[-1] - 1):",
+     [(P, "test_head_mean_exposure_eq5", ())]),
+    ("eq6_divides_by_T", "core.py", "return 100.0 * total / (T - 1)", "return 100.0 * total / T",
+     [(P, "test_adjacent_ref_mass_change_eq6", ())]),
+    ("eq6_signed_change", "core.py", "total = total + np.abs(Mbar[t] - Mbar[t - 1])",
+     "total = total + (Mbar[t] - Mbar[t - 1])",
+     [(P, "test_adjacent_ref_mass_change_eq6", ())]),
+    ("eq6_fraction_not_points", "core.py", "return 100.0 * total / (T - 1)", "return total / (T - 1)",
+     [(P, "test_adjacent_ref_mass_change_eq6", ())]),
     # gate, Eqs. 12-13 and the bounded-age refresh (core.py)
     ("gate_mean_then_product", "core.py",
      "g = [float(D[s][h]) * float(M_prev[s][h]) for h in range(len(D[s]))]",

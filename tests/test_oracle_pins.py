@@ -529,3 +529,31 @@ def test_sampled_rows_change_ignores_unsampled_rows():
     np.testing.assert_allclose(rec[1][0]["D"], want, rtol=1e-12)
     full = oracle.closed_loop(lambda t, b: bits[t], 2, 1, B, theta=1e9, delta_max=10)
     assert np.abs(full[1][0]["D"] - want).max() > 1e-2
+
+
+def test_head_mean_exposure_eq5():
+    """Eq. 5 is the plain mean over the head axis (the last one)."""
+    M = np.array([[[0.1, 0.3, 0.2, 0.0]], [[0.5, 0.5, 0.5, 0.5]]])  # [T=2, B=1, H=4]
+    got = oracle.head_mean_exposure(M)
+    assert got.shape == (2, 1)
+    assert got[0, 0] == pytest.approx(0.15) and got[1, 0] == pytest.approx(0.5)
+    # one head: the mean is that head's exposure
+    assert oracle.head_mean_exposure([[0.37]])[0] == pytest.approx(0.37)
+
+
+def test_adjacent_ref_mass_change_eq6():
+    """Eq. 6 in percentage points: 100/(T-1) times the summed absolute step-to-step
+    change. Closed forms: a constant series gives 0, a linear ramp of slope c
+    gives 100|c| whatever T, and a zig-zag counts every change with its size."""
+    assert oracle.adjacent_ref_mass_change([0.2, 0.2, 0.2, 0.2]) == pytest.approx(0.0)
+    for T in (2, 5, 9):
+        up = [0.10 + 0.003 * t for t in range(T)]
+        assert oracle.adjacent_ref_mass_change(up) == pytest.approx(0.3)
+        assert oracle.adjacent_ref_mass_change(up[::-1]) == pytest.approx(0.3)
+    # 0.10 -> 0.12 -> 0.11: (0.02 + 0.01) / 2 steps = 1.5 points (dividing by T would give 1.0)
+    assert oracle.adjacent_ref_mass_change([0.10, 0.12, 0.11]) == pytest.approx(1.5)
+    # per block and sample: the first axis is the step axis
+    got = oracle.adjacent_ref_mass_change(np.array([[0.1, 0.4], [0.2, 0.4], [0.1, 0.1]]))
+    assert got == pytest.approx([10.0, 15.0])
+    with pytest.raises(ValueError):
+        oracle.adjacent_ref_mass_change([0.1])
