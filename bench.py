@@ -93,9 +93,11 @@ EXEC_OPTS = {"fused_cache": True}
 
 
 def launches_per_block(t):
-    """Kernels one block of step t launches: Q change (t >= 1), gate,
-    attention, and the cache update unless it is fused into the attention."""
-    return (1 if t >= 1 else 0) + 2 + (0 if EXEC_OPTS["fused_cache"] else 1)
+    """Kernels one block of step t launches: the gate (t = 0) or the Q change
+    with the gate in the same launch (t >= 1; the Q change's cluster path,
+    which every workload here takes), the attention, and the cache update
+    unless it is fused into the attention."""
+    return 2 + (0 if EXEC_OPTS["fused_cache"] else 1)
 
 
 # ----------------------------------------------------------------------------- helpers
@@ -713,16 +715,28 @@ def time_e2e(wl, inputs, warmup, steps, keep=None):
                                           "them, no pinned range set aside"}}
 
 
-def _q_delta_launch_ms(pairs, B, H, eps, reps):
+def _q_delta_launch_ms(pairs, B, H, eps, reps, gate_mpl=0):
     """Average duration of one refadapt_q_delta launch over `reps` launches
     rotating over `pairs` (current, previous), queued behind a GPU-side sleep
-    so they run back to back; the best of three runs."""
+    so they run back to back; the best of three runs. gate_mpl > 0 times
+    refadapt_q_delta_gate instead (the gate of block 0, step 1, on mass
+    partials of that length), the call the executor makes."""
     import torch
     from paper_2609_32415_gb300 import api
     ws = api.q_delta_workspace(B, H)
     out = torch.empty((B, H), dtype=torch.float32, device="cuda")
+    if gate_mpl > 0:
+        state = api.new_state(B, "cuda")
+        mode = torch.zeros(B, dtype=torch.int32, device="cuda")
+        mass = torch.full((B, H, gate_mpl), 0.01, dtype=torch.float32, device="cuda")
+
+        def call(a, b):
+            api.refadapt_q_delta_gate(a, b, out, ws, 1, 0, state, mode, 0.1, 1000, mass, 128 * gate_mpl, eps)
+    else:
+        def call(a, b):
+            api.refadapt_q_delta(a, b, out, ws, eps)
     for a, b in pairs:                           # warm-up
-        api.refadapt_q_delta(a, b, out, ws, eps)
+        call(a, b)
     runs = []
     for _ in range(3):
         torch.cuda.synchronize()
@@ -731,7 +745,7 @@ def _q_delta_launch_ms(pairs, B, H, eps, reps):
         e0.record()
         for i in range(reps):
             a, b = pairs[i % len(pairs)]
-            api.refadapt_q_delta(a, b, out, ws, eps)
+            call(a, b)
         e1.record()
         torch.cuda.synchronize()
         runs.append(e0.elapsed_time(e1) / reps)
@@ -776,6 +790,9 @@ def time_q_delta(wl, inputs, reps=64):
         cur = (prev.float() + 0.3 * torch.randn(shape, generator=g, device="cuda") / wl.d ** 0.5).to(torch.bfloat16)
         pairs.append((cur, prev))
     ms = _q_delta_launch_ms(pairs, wl.B, wl.H, wl.eps, reps)
+    from paper_2609_32415_gb300 import api
+    ms_gate = _q_delta_launch_ms(pairs, wl.B, wl.H, wl.eps, reps,
+                                 gate_mpl=api.refadapt_mass_partial_len(wl.n_text, wl.n_tgt))
     byts = 4 * wl.n_tgt * wl.H * wl.d * wl.B
     # Context: a library streaming read of the same number of bytes (torch's
     # sum over one contiguous buffer), timed the same way.
@@ -792,7 +809,8 @@ def time_q_delta(wl, inputs, reps=64):
         torch.cuda.synchronize()
         lib_runs.append(e0.elapsed_time(e1) / reps)
     del bufs
-    return {"bytes": byts, "ms": ms, "gbs": byts / ms / 1e6, "lib_read_gbs": byts / min(lib_runs) / 1e6}
+    return {"bytes": byts, "ms": ms, "gbs": byts / ms / 1e6, "lib_read_gbs": byts / min(lib_runs) / 1e6,
+            "ms_with_gate": ms_gate}
 
 
 def cpu_oracle_sample(wl, X, budget_s):
@@ -863,6 +881,7 @@ def q_delta_summary(qd, peaks):
             "peak": peaks["hbm_gbs"], "unit": "GB/s", "frac": round(qd["gbs"] / peaks["hbm_gbs"], 4),
             "bytes_per_launch": qd["bytes"], "launch_ms": round(qd["ms"], 5),
             "same_bytes_torch_sum_gbs": round(qd["lib_read_gbs"], 1),
+            "with_gate_launch_ms": round(qd["ms_with_gate"], 5),
             "peak_kind": "%s HBM copy" % peaks["source"]}
 
 

@@ -291,6 +291,26 @@ typedef enum { RA_CUE_PRODUCT = 0, RA_CUE_CHANGE = 1, RA_CUE_EXPOSURE = 2 } ra_c
 
 ra_status refadapt_gate(const ra_gate_args* args, void* stream);
 
+/* refadapt_q_delta_gate — refadapt_q_delta, then refadapt_gate on the D it
+ * produced (paper Eq. 1, then Eqs. 12-13 / App. A.2 / Algorithm 1), with the
+ * results of the two calls, bit for bit. When the Q change takes its cluster
+ * path this is one launch: each cluster's leader writes its slab's D and takes
+ * a ticket from the workspace; the leader that takes the last one runs the
+ * decision on all B x H values in its CTA. No CTA waits for another. On the
+ * multi-block path the gate is a second launch behind the Q change.
+ *
+ *  q_cur ... workspace_bytes   as for refadapt_q_delta (the workspace also
+ *                              holds the ticket; same size function).
+ *  gate                        as for refadapt_gate with gate->B == B,
+ *                              gate->H == H, gate->t >= 1 (step 0 has no Q
+ *                              change: call refadapt_gate), and gate->q_delta
+ *                              NULL or equal to d_out.
+ * Errors: RA_EINVAL for either call's argument errors, nothing queued.
+ */
+ra_status refadapt_q_delta_gate(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
+                                float eps, float* d_out, void* workspace, size_t workspace_bytes,
+                                const ra_gate_args* gate, void* stream);
+
 /* ------------------------------------------------------------------ cache
  * refadapt_ref_cache_update — materialise a block's reference K/V into its
  * cache slot (paper Eq. 11, Z_b = (H_b, K_b, V_b, a_b); Algorithm 1: a

@@ -23,7 +23,7 @@ EXPORTED = (
     "refadapt_ref_cache_update", "refadapt_status_string", "refadapt_last_error",
     "refadapt_set_wait_budget_ns", "refadapt_check_error", "refadapt_version",
     "refadapt_selftest_wait_timeout", "refadapt_q_delta_noalloc", "refadapt_rope_table",
-    "refadapt_ln_modulate", "refadapt_gemm",
+    "refadapt_ln_modulate", "refadapt_gemm", "refadapt_q_delta_gate",
 )
 RA_EPI_STORE, RA_EPI_GELU, RA_EPI_RESID, RA_EPI_QKV = 0, 1, 2, 3
 
@@ -118,6 +118,9 @@ def load():
     lib.refadapt_state_init.argtypes = [c_void_p, c_int32, c_void_p]
     lib.refadapt_gate.restype = c_int32
     lib.refadapt_gate.argtypes = [POINTER(RaGateArgs), c_void_p]
+    lib.refadapt_q_delta_gate.restype = c_int32
+    lib.refadapt_q_delta_gate.argtypes = [POINTER(RaSeg), POINTER(RaSeg), c_int32, c_int32, c_int32, c_float,
+                                          c_void_p, c_void_p, c_size_t, POINTER(RaGateArgs), c_void_p]
     lib.refadapt_ref_cache_update.restype = c_int32
     lib.refadapt_ref_cache_update.argtypes = [POINTER(RaSeg), POINTER(RaSeg), POINTER(RaSeg), POINTER(RaSeg),
                                               c_int32, c_int32, c_int32, POINTER(RaSeg), POINTER(RaSeg),

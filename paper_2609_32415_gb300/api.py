@@ -126,8 +126,8 @@ def new_state(B, device="cuda", stream=None):
     return st
 
 
-def refadapt_gate(t, b, state, mode_out, theta, delta_max, B, H, q_delta=None, mass_partial_prev=None,
-                  mass_row_count=0, forced_boundary=-1, gbar_out=None, m_out=None, cue=0, stream=None):
+def _gate_args(t, b, state, mode_out, theta, delta_max, B, H, q_delta, mass_partial_prev, mass_row_count,
+               forced_boundary, gbar_out, m_out, cue):
     a = RaGateArgs()
     a.theta = float(theta)
     a.t, a.b, a.B, a.H = int(t), int(b), int(B), int(H)
@@ -142,7 +142,29 @@ def refadapt_gate(t, b, state, mode_out, theta, delta_max, B, H, q_delta=None, m
     a.mode_out = _ptr(mode_out)
     a.gbar_out = _ptr(gbar_out)
     a.m_out = _ptr(m_out)
+    return a
+
+
+def refadapt_gate(t, b, state, mode_out, theta, delta_max, B, H, q_delta=None, mass_partial_prev=None,
+                  mass_row_count=0, forced_boundary=-1, gbar_out=None, m_out=None, cue=0, stream=None):
+    a = _gate_args(t, b, state, mode_out, theta, delta_max, B, H, q_delta, mass_partial_prev, mass_row_count,
+                   forced_boundary, gbar_out, m_out, cue)
     return check("refadapt_gate", _lib.load().refadapt_gate(ctypes.byref(a), _stream(stream)))
+
+
+def refadapt_q_delta_gate(q_cur, q_prev, d_out, workspace, t, b, state, mode_out, theta, delta_max,
+                          mass_partial_prev, mass_row_count, eps=1e-6, forced_boundary=-1, gbar_out=None,
+                          m_out=None, cue=0, stream=None):
+    """refadapt_q_delta then refadapt_gate on its D (t >= 1), in one launch
+    when the Q change takes its cluster path."""
+    lib = _lib.load()
+    B, H, _, d = q_cur.shape
+    sc, sp = seg(q_cur), seg(q_prev)
+    a = _gate_args(t, b, state, mode_out, theta, delta_max, B, H, d_out, mass_partial_prev, mass_row_count,
+                   forced_boundary, gbar_out, m_out, cue)
+    return check("refadapt_q_delta_gate", lib.refadapt_q_delta_gate(
+        ctypes.byref(sc), ctypes.byref(sp), B, H, d, float(eps), _ptr(d_out), _ptr(workspace),
+        workspace.numel() * workspace.element_size(), ctypes.byref(a), _stream(stream)))
 
 
 def refadapt_ref_cache_update(k_src, v_src, k_cache, v_cache, mode, t, a_b=None, x_src=None, x_cache=None,

@@ -38,6 +38,15 @@
 // slab in unit order into one slot per (slab, CTA) of the workspace; the
 // slab's last contributor (ticket counter) adds the slots in CTA order,
 // writes D and re-arms the counter.
+//
+// refadapt_q_delta_gate runs Algorithm 1's gate on the new D in the same
+// launch (cluster path): each leader's first consumer warp reduces its
+// slab's mass partials of the previous step into M right after the
+// dependency wait (while the first units are in flight); after D, the leader
+// stores its head's score term and takes a ticket, and the leader that takes
+// the last one sums the B x H terms in head order and decides (gate_body.cuh;
+// the same arithmetic and order as refadapt_gate). On the multi-block path
+// the gate is a launch of its own.
 #include <cuda.h>
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
@@ -47,6 +56,7 @@
 #include <mutex>
 
 #include "api_common.h"
+#include "gate_body.cuh"
 #include "tc_ptx.cuh"
 
 namespace ra {
@@ -317,6 +327,11 @@ struct ClusterParams {
   float eps;
   float* d_out;
   uint64_t budget_ns;
+  // refadapt_q_delta_gate: the last cluster to write its D runs the gate
+  int32_t fuse_gate;
+  uint32_t* gate_ticket;  // workspace counter (zero between launches)
+  float2* gate_terms;     // workspace [B * H]: each head's score term (g, e)
+  gate::Params gp;        // gp.qd == d_out
 };
 
 __device__ __forceinline__ void cluster_sync_all() {
@@ -349,6 +364,8 @@ __global__ void __launch_bounds__(ClLayout<S, UB>::THREADS)
   const int k0 = p.k_begin[rank];
   const int nu = p.k_begin[rank + 1] - k0;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  float m_exp = 0.f;  // fused gate: M_{t-1,b,h} of this slab (leader, thread 0)
+  float d_val = 0.f;  // the slab's D (leader, thread 0)
   // This CTA has started (its shared memory exists): the remote stores at the
   // end wait for every CTA's arrival, the loads below need no one else.
   cluster_arrive();
@@ -422,6 +439,10 @@ __global__ void __launch_bounds__(ClLayout<S, UB>::THREADS)
     // ------------------------------------------------------------ consumers
     named_bar_sync(2, L::THREADS);  // the ring's barriers are initialised
     asm volatile("griddepcontrol.wait;" ::: "memory");  // orders the final store of D
+    // Fused gate: the leader's first warp reduces this slab's mass partials of
+    // the previous step (they need nothing of this launch) while the first
+    // units are still on their way.
+    if (p.fuse_gate && rank == 0 && warp == 0) m_exp = gate::head_exposure(p.gp, b * p.H + h);
     float dh = 0.f, dl = 0.f, ph = 0.f, pl = 0.f;  // this warp's units, in order (lane 0)
     for (int i = warp; i < nu; i += CL_CONSUMERS) {
       const int s = i % CL_STAGES;
@@ -486,7 +507,41 @@ __global__ void __launch_bounds__(ClLayout<S, UB>::THREADS)
       ff_add(ph, pl, v.z);
       pl += v.w;
     }
-    p.d_out[b * p.H + h] = sqrtf(dh + dl) / (sqrtf(ph + pl) + p.eps);
+    d_val = sqrtf(dh + dl) / (sqrtf(ph + pl) + p.eps);
+    p.d_out[b * p.H + h] = d_val;
+  }
+  if (p.fuse_gate && rank == 0) {
+    // Every leader publishes its head's score term (and M for the log), then
+    // a ticket after a fence; the leader that takes the last ticket re-arms
+    // the counter and its CTA sums the terms in head order and decides (the
+    // arithmetic of refadapt_gate, in its order). No CTA waits for another.
+    volatile int32_t* last = reinterpret_cast<volatile int32_t*>(smem + L::OFF_MISC + 4);
+    volatile int32_t* full_step = last + 1;
+    if (threadIdx.x == 0) {
+      const int sh = b * p.H + h;
+      float g, e;
+      gate::score_term(p.gp.cue, d_val, m_exp, g, e);
+      p.gate_terms[sh] = make_float2(g, e);
+      if (p.gp.m_out) p.gp.m_out[sh] = m_exp;
+      __threadfence();
+      const uint32_t total = gridDim.y * gridDim.z;
+      const bool is_last = atomicAdd(p.gate_ticket, 1u) == total - 1;
+      if (is_last) {
+        *p.gate_ticket = 0u;  // re-armed for the next launch (visible when this one completes)
+        *full_step = gate::open_step(p.gp);
+      }
+      *last = is_last ? 1 : 0;
+    }
+    __syncthreads();
+    if (*last) {
+      const float2* terms = p.gate_terms;
+      for (int s = threadIdx.x; s < p.gp.B; s += blockDim.x)
+        gate::decide_sample(p.gp, s, *full_step, true, [&](int hh, float& g, float& e) {
+          const float2 v = __ldcg(terms + s * p.gp.H + hh);
+          g = v.x;
+          e = v.y;
+        });
+    }
   }
 }
 
@@ -559,7 +614,8 @@ extern "C" size_t refadapt_q_delta_workspace_size(int32_t B, int32_t H) {
   if (B < 1 || H < 1) return 0;
   const size_t bh = size_t(B) * size_t(H);
   const size_t counters = ((bh * sizeof(uint32_t)) + 255) / 256 * 256;
-  return counters + bh * ra::qd::MAX_SPLITS * sizeof(float4);
+  // refadapt_q_delta_gate: the heads' score terms and a ticket counter
+  return counters + bh * ra::qd::MAX_SPLITS * sizeof(float4) + (bh * sizeof(float2) + 255) / 256 * 256 + 256;
 }
 
 namespace ra {
@@ -602,8 +658,11 @@ ra_status validate(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, i
 // validate(). The workspace is touched only by the multi-block path; with
 // clear_counters its ticket counters are zeroed on the stream right before
 // that kernel (for a workspace whose earlier contents are unknown).
+// With `fuse` (refadapt_q_delta_gate) the gate runs on the new D: inside the
+// cluster kernel, or as its own launch behind the multi-block kernel.
 ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H, int32_t d,
-                 float eps, float* d_out, void* workspace, bool clear_counters, void* stream) {
+                 float eps, float* d_out, void* workspace, bool clear_counters, void* stream,
+                 const gate::Params* fuse = nullptr) {
   const int n = q_cur->n;
   const int bh = B * H;
   {
@@ -657,6 +716,14 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
       c.eps = eps;
       c.d_out = d_out;
       c.budget_ns = wait_budget_ns();
+      if (fuse) {
+        const size_t counters = ((size_t(bh) * sizeof(uint32_t)) + 255) / 256 * 256;
+        char* tail = static_cast<char*>(workspace) + counters + size_t(bh) * MAX_SPLITS * sizeof(float4);
+        c.fuse_gate = 1;
+        c.gate_terms = reinterpret_cast<float2*>(tail);
+        c.gate_ticket = reinterpret_cast<uint32_t*>(tail + (size_t(bh) * sizeof(float2) + 255) / 256 * 256);
+        c.gp = *fuse;
+      }
       if (!c.bulk && (!encode_seg(&c.tm_c, *q_cur, B, H, d, d, rows_per_unit, false) ||
                       !encode_seg(&c.tm_p, *q_prev, B, H, d, d, rows_per_unit, false)))
         return RA_EINVAL;
@@ -737,7 +804,9 @@ ra_status launch(const char* who, const ra_seg* q_cur, const ra_seg* q_prev, int
     }
   }
   q_delta_kernel<<<p.grid, THREADS, SMEM_ALLOC, static_cast<cudaStream_t>(stream)>>>(p);
-  return launch_status(who);
+  const ra_status ls = launch_status(who);
+  if (ls != RA_OK || !fuse) return ls;
+  return gate::launch(*fuse, static_cast<cudaStream_t>(stream), who);
 }
 
 }  // namespace qd
@@ -758,6 +827,36 @@ extern "C" ra_status refadapt_q_delta(const ra_seg* q_cur, const ra_seg* q_prev,
     return RA_EINVAL;
   }
   return qd::launch(who, q_cur, q_prev, B, H, d, eps, d_out, workspace, false, stream);
+}
+
+extern "C" ra_status refadapt_q_delta_gate(const ra_seg* q_cur, const ra_seg* q_prev, int32_t B, int32_t H,
+                                           int32_t d, float eps, float* d_out, void* workspace,
+                                           size_t workspace_bytes, const ra_gate_args* gate, void* stream) {
+  using namespace ra;
+  clear_error();
+  const char* who = "refadapt_q_delta_gate";
+  const ra_status v = qd::validate(who, q_cur, q_prev, B, H, d, eps, d_out);
+  if (v != RA_OK) return v;
+  if (!workspace || reinterpret_cast<uintptr_t>(workspace) % 16 != 0 ||
+      workspace_bytes < refadapt_q_delta_workspace_size(B, H)) {
+    set_error("%s: workspace must be non-NULL, 16-byte aligned and >= %zu bytes", who,
+              refadapt_q_delta_workspace_size(B, H));
+    return RA_EINVAL;
+  }
+  if (!gate) {
+    set_error("%s: gate args are NULL", who);
+    return RA_EINVAL;
+  }
+  if (gate->B != B || gate->H != H || gate->t < 1 || (gate->q_delta && gate->q_delta != d_out)) {
+    set_error("%s: the gate's B, H must match, t must be >= 1 and q_delta must be NULL or d_out", who);
+    return RA_EINVAL;
+  }
+  ra_gate_args ga = *gate;
+  ga.q_delta = d_out;
+  gate::Params gp;
+  const ra_status gv = gate::make_params(&ga, who, &gp);
+  if (gv != RA_OK) return gv;
+  return qd::launch(who, q_cur, q_prev, B, H, d, eps, d_out, workspace, false, stream, &gp);
 }
 
 // ---------------------------------------------------------------------------

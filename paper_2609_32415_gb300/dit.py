@@ -120,14 +120,15 @@ class DiTExecutor:
             for r in ("text", "tgt")], 3 * C, C, RA_EPI_QKV, rope=self.rope, H=self.H, d=self.d,
             norm_eps=self.norm_eps, err_word=self.err, stream=stream)
         # 2. Q change and the gate
-        have_prev = t >= 1
-        if have_prev:
-            api.refadapt_q_delta(cur, prev, self.D[b], self.workspace, self.eps, stream)
-        api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
-                          q_delta=self.D[b] if have_prev else None,
-                          mass_partial_prev=self.mass[b] if have_prev else None,
-                          mass_row_count=self.mass_row_count, forced_boundary=self.forced_boundary,
-                          gbar_out=self.gbar[li, b], m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
+        if t >= 1:
+            api.refadapt_q_delta_gate(cur, prev, self.D[b], self.workspace, t, b, self.state, mode, self.theta,
+                                      self.delta_max, self.mass[b], self.mass_row_count, eps=self.eps,
+                                      forced_boundary=self.forced_boundary, gbar_out=self.gbar[li, b],
+                                      m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
+        else:
+            api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
+                              mass_row_count=self.mass_row_count, forced_boundary=self.forced_boundary,
+                              gbar_out=self.gbar[li, b], m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
         # 3. reference rows (gated on the mode): LN of H_b, QKV into the cache slot
         api.refadapt_ln_modulate(
             [{"h": hin["ref"], "x": self.x["ref"], "shift": ms["ref"]["shift_a"], "scale": ms["ref"]["scale_a"],

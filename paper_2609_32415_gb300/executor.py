@@ -172,15 +172,18 @@ class Executor:
         mode = self.modes[li, b]
         have_prev = t >= 1 and self._prev_qtgt[b] is not None
         if have_prev:
+            # Eq. 1 and the decision in one call (one launch on the cluster path)
             ref_q = self.anchor[b] if self.anchor is not None else self._prev_qtgt[b]
             k = self.sample_stride
-            api.refadapt_q_delta(qt[:, :, ::k, :] if k > 1 else qt, ref_q[:, :, ::k, :] if k > 1 else ref_q,
-                                 self.D[b], self.workspace, self.eps, stream)
-        api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
-                          q_delta=self.D[b] if have_prev else None,
-                          mass_partial_prev=self.mass[b] if have_prev else None,
-                          mass_row_count=self.mass_row_count, forced_boundary=self.forced_boundary,
-                          gbar_out=self.gbar[li, b], m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
+            api.refadapt_q_delta_gate(qt[:, :, ::k, :] if k > 1 else qt, ref_q[:, :, ::k, :] if k > 1 else ref_q,
+                                      self.D[b], self.workspace, t, b, self.state, mode, self.theta,
+                                      self.delta_max, self.mass[b], self.mass_row_count, eps=self.eps,
+                                      forced_boundary=self.forced_boundary, gbar_out=self.gbar[li, b],
+                                      m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
+        else:
+            api.refadapt_gate(t, b, self.state, mode, self.theta, self.delta_max, self.B, self.H,
+                              mass_row_count=self.mass_row_count, forced_boundary=self.forced_boundary,
+                              gbar_out=self.gbar[li, b], m_out=self.M[li, b], cue=CUES[self.cue], stream=stream)
         if self.anchor is not None:
             # Materialising blocks move their anchor to this step's target Q (the
             # V copy is skipped: source and destination coincide).
