@@ -1,8 +1,10 @@
 """Algorithm 1's host loop over the C ABI: one denoising step = for each block,
 Q change -> gate -> cache materialisation -> joint attention, enqueued with the
-decisions kept on the device (no host sync inside a step). By default a block's
-decision and cache update run on a side stream beside the previous block's
-attention, and consecutive attentions alternate between two streams (see
+decisions kept on the device (no host sync inside a step). The Q change and the
+gate are one launch from step 1 on (refadapt_q_delta_gate); the cache
+materialisation rides in the attention (fused_cache). By default a block's
+decision runs on a side stream beside the previous block's attention, and
+consecutive attentions alternate between two streams (see
 Executor.step); overlap=False keeps every launch on the caller's stream.
 
 Per block b the executor owns the cache state of paper Eq. 11: reference K and
@@ -62,9 +64,10 @@ class Executor:
     rows only. k = 1 uses every row.
 
     ``overlap`` (default) runs step() on three streams of its own (a side
-    stream for the decisions and cache updates, two higher-priority streams
-    for the attentions), forked from and joined to the caller's stream per
-    step; the results equal the one-stream order bit for bit.
+    stream for the decisions, and the cache updates when they are not fused;
+    two higher-priority streams for the attentions), forked from and joined
+    to the caller's stream per step; the results equal the one-stream order
+    bit for bit.
 
     ``fused_cache`` (default) lets the attention of a materialising block
     write its cache slot (refadapt_joint_attn's ref_fresh arguments) instead
@@ -101,9 +104,9 @@ class Executor:
         self.M = torch.zeros((self.log_steps, n_blocks, B, H), dtype=torch.float32, device=dev)
         self.workspace = api.q_delta_workspace(B, H, dev)
         self.state = api.new_state(B, dev)
-        # overlap: step() runs each block's decision (Q change, gate) and cache
-        # update on a side stream one block ahead, in the previous attention's
-        # tail wave (SMs its last wave leaves idle); see step().
+        # overlap: step() runs each block's decision (Q change with the gate)
+        # on a side stream one block ahead, in the previous attention's tail
+        # wave (SMs its last wave leaves idle); see step().
         self.overlap = bool(overlap)
         self.fused_cache = bool(fused_cache)
         if self.overlap:
@@ -251,17 +254,19 @@ class Executor:
         outs[b] (optional): dict role -> O. The caller keeps step t's target Q
         alive until step t + 1 has been enqueued (it is read as q_{t-1}).
 
-        With overlap (the default) block b's decision (Q change, gate) and
-        cache update run on a side stream, ordered after the step's start and
-        after the attention of block b - 2, and block b's attention waits for
-        them: so they run during the attention of block b - 1, whose last wave
+        With overlap (the default) block b's decision (the Q change with the
+        gate; the cache update too when it is not fused into the attention)
+        runs on a side stream, ordered after the step's start and after the
+        attention of block b - 2, and block b's attention waits for it: so it
+        runs during the attention of block b - 1, whose last wave
         leaves SMs idle (the attentions run on higher-priority streams, so
         their pending CTAs go first). Consecutive attentions alternate between
         two streams: they share no data (inputs, cache slot, outputs and mass
         partials are the block's own), so block b + 1's first CTAs may start in
         block b's last wave. Every stream forks from the caller's stream at
-        the step's start and joins it at the end. A gate reads only its block's target queries, the
-        block's previous-step mass partials and the controller state of the
+        the step's start and joins it at the end. A gate reads only its
+        block's target queries, the block's previous-step mass partials and
+        the controller state of the
         blocks before it, never an attention of the same step, so the results
         are those of the one-stream order. Every event is recorded inside the
         step, which can be captured as a CUDA graph."""
