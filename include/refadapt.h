@@ -158,7 +158,7 @@ typedef struct {
   const int32_t* mode;
   float* mass_partial;
   int32_t* err_word;
-  ra_seg ref_fresh_q, ref_fresh_k, ref_fresh_v;  /* fused cache update; ref_fresh_k.ptr NULL = off */
+  ra_seg ref_fresh_q, ref_fresh_k, ref_fresh_v;  /* fused cache update; off when these ptrs and a_b are NULL */
   int32_t* a_b;
   int32_t step;
   int32_t reserved;  /* set to 0 */
