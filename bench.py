@@ -82,14 +82,20 @@ def parse_args():
     ap.add_argument("--separate-cache-update", action="store_true",
                     help="refresh each materialising block's cache slot with its own refadapt_ref_cache_update "
                          "launch before the attention instead of inside it")
+    ap.add_argument("--trace", default=None,
+                    help="write the main trajectory's observation record (per step and block: modes, gbar, the "
+                         "exposure the gate read, a_b) as JSON lines to this file, after the timed region")
+    ap.add_argument("--nvtx", action="store_true",
+                    help="NVTX ranges around every block's decision and attention (for timeline profilers)")
     ap.add_argument("--out", default=None, help="also write the JSON line to this file")
     args = ap.parse_args()
     EXEC_OPTS["fused_cache"] = not args.separate_cache_update
+    EXEC_OPTS["nvtx"] = bool(args.nvtx)
     return args
 
 
 # Executor options every timed schedule shares (set from the command line).
-EXEC_OPTS = {"fused_cache": True}
+EXEC_OPTS = {"fused_cache": True, "nvtx": False}
 
 
 def launches_per_block(t):
@@ -318,7 +324,8 @@ def union_length(intervals):
 
 
 def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False, clocks=None,
-                    barrier=None, cue="product", theta=None, diagnostics=False, diag_row_stride=8, overlap=True):
+                    barrier=None, cue="product", theta=None, diagnostics=False, diag_row_stride=8, overlap=True,
+                    trace_path=None):
     """Run warmup + timed steps (cycling the trajectory); returns timing dict.
     overlap=False keeps every launch of a step on one stream in Algorithm 1's
     block order (each block's Q change, gate, cache update, then attention):
@@ -372,6 +379,10 @@ def time_trajectory(wl, inputs, warmup, steps, delta_max=None, attn_timing=False
         barrier()
     ex.attn_hook = None
     ex.check()
+    if trace_path:
+        with open(trace_path, "w") as f:
+            for rec in ex.trace(wl.n_steps):
+                f.write(json.dumps(rec) + "\n")
     total_ms = step_ev[0].elapsed_time(step_ev[-1])
     per_step = [step_ev[k].elapsed_time(step_ev[k + 1]) for k in range(steps)]
     modes = ex.modes.cpu().numpy()
@@ -936,7 +947,7 @@ def main_ours(args):
     torch.cuda.synchronize()
     clocks = Clocks(local)
     main = time_trajectory(wl, inputs, args.warmup, args.steps, attn_timing=True, clocks=clocks,
-                           barrier=barrier)
+                           barrier=barrier, trace_path=args.trace if rank == 0 else None)
     total_ms = reduce_max_ms(main["total_ms"], device="cuda")
     ms_per_step = job_ms_per_step(total_ms, args.steps, ws)
     refresh = None

@@ -16,6 +16,8 @@ reference rows, and the joint-attention kernel copies them into the slot in
 the same pass (fused_cache, the default); fused_cache=False refreshes the slot
 with refadapt_ref_cache_update first and the attention reads the slot.
 """
+import contextlib
+
 import torch
 
 from . import api
@@ -77,7 +79,7 @@ class Executor:
     def __init__(self, n_blocks, B, H, d, n_text, n_ref, n_tgt, theta, delta_max, eps=1e-6,
                  mass_rows=0, forced_boundary=-1, softmax_scale=0.0, bias=None, log_steps=8,
                  device="cuda", cue="product", diagnostics=False, diag_row_stride=1, sample_stride=1,
-                 overlap=True, fused_cache=True):
+                 overlap=True, fused_cache=True, nvtx=False):
         if cue not in CUES:
             raise ValueError("unknown cue %r" % (cue,))
         self.cue = cue
@@ -146,6 +148,12 @@ class Executor:
                               "tgt": torch.empty((B, H, n_s, d), dtype=torch.bfloat16, device=dev)} for _ in range(2)]
         self._out = [None, None]
         self.attn_hook = None   # optional callable(phase in {"pre", "post"}, t, b), e.g. CUDA events
+        self.nvtx = bool(nvtx)
+
+    def _range(self, name):
+        """An NVTX range around the launches it encloses (nvtx=True), for
+        timeline profilers; nothing otherwise."""
+        return torch.cuda.nvtx.range(name) if self.nvtx else contextlib.nullcontext()
 
     def scratch_outputs(self, parity=0):
         """A set of O buffers (text, ref, tgt) reused by every block of one
@@ -174,6 +182,11 @@ class Executor:
         li = (t % self.log_steps) if log_index is None else log_index
         mode = self.modes[li, b]
         have_prev = t >= 1 and self._prev_qtgt[b] is not None
+        with self._range("t%d b%d decision" % (t, b)):
+            self._decide(t, b, qt, li, mode, have_prev, stream)
+        self._prev_qtgt[b] = qt
+
+    def _decide(self, t, b, qt, li, mode, have_prev, stream):
         if have_prev:
             # Eq. 1 and the decision in one call (one launch on the cluster path)
             ref_q = self.anchor[b] if self.anchor is not None else self._prev_qtgt[b]
@@ -192,7 +205,6 @@ class Executor:
             # V copy is skipped: source and destination coincide).
             an = self.anchor[b]
             api.refadapt_ref_cache_update(qt, an, an, an, mode, t, None, stream=stream)
-        self._prev_qtgt[b] = qt
 
     def attend_block(self, t, b, x, out, log_index=None, stream=None):
         """The attention half of block b of step t, after gate_block(t, b): the
@@ -222,6 +234,14 @@ class Executor:
         qt = x["tgt"][0]
         if self.attn_hook is not None:
             self.attn_hook("pre", t, b)
+        with self._range("t%d b%d attention" % (t, b)):
+            self._attend(t, b, x, out, mode, qt, stream)
+        if self.attn_hook is not None:
+            self.attn_hook("post", t, b)
+        if self.diagnostics:
+            self._diagnose(t, b, li, x, out, stream)
+
+    def _attend(self, t, b, x, out, mode, qt, stream):
         api.refadapt_joint_attn(
             (x["text"][0], self.cache_x[b], qt),
             (x["text"][1], self.cache_k[b], x["tgt"][1]),
@@ -231,10 +251,6 @@ class Executor:
             mass_rows=self.mass_rows, err_word=self.err, mass_row_stride=self.sample_stride,
             ref_fresh=x["ref"] if self.fused_cache else None,
             a_b=self.a_b[b] if self.fused_cache else None, step=t, stream=stream)
-        if self.attn_hook is not None:
-            self.attn_hook("post", t, b)
-        if self.diagnostics:
-            self._diagnose(t, b, li, x, out, stream)
 
     def _diagnose(self, t, b, li, x, out, stream):
         k = self.diag_row_stride
@@ -345,6 +361,65 @@ class Executor:
         Mbar = M.mean(axis=-1)
         Delta = 100.0 * np.abs(np.diff(Mbar, axis=0)).sum(axis=0) / (T - 1)
         return Mbar, Delta
+
+    # Cross-step state of Algorithm 1 (Eq. 11's block caches and a_b, the
+    # controller state, the previous step's mass partials and Q change) and the
+    # per-step logs; the Q-change workspace is zero between calls and is not
+    # state.
+    _STATE = ("cache_k", "cache_v", "cache_x", "a_b", "mass", "D", "state", "modes", "gbar", "M")
+    _STATE_OPT = ("anchor", "E_K", "E_V", "I_KV", "M_fresh_part")
+
+    def snapshot(self):
+        """A host copy of everything a trajectory carries from one step to
+        the next (after the enqueued work has finished): restore() on an
+        executor of the same configuration continues the trajectory with the
+        same results, bit for bit. The previous step's target queries are
+        copied too (the next step's Q change reads them)."""
+        torch.cuda.synchronize(self.cache_k.device)
+        snap = {k: getattr(self, k).detach().cpu().clone() for k in self._STATE}
+        for k in self._STATE_OPT:
+            if getattr(self, k, None) is not None:
+                snap[k] = getattr(self, k).detach().cpu().clone()
+        snap["prev_qtgt"] = [None if q is None else q.detach().cpu().clone() for q in self._prev_qtgt]
+        snap["config"] = self._config()
+        return snap
+
+    def restore(self, snap):
+        """Load a snapshot() taken from an executor of the same configuration."""
+        if snap["config"] != self._config():
+            raise ValueError("restore: the snapshot's configuration differs: %r vs %r"
+                             % (snap["config"], self._config()))
+        for k in self._STATE + self._STATE_OPT:
+            if k in snap:
+                getattr(self, k).copy_(snap[k])
+        dev = self.cache_k.device
+        self._prev_qtgt = [None if q is None else q.to(dev) for q in snap["prev_qtgt"]]
+        torch.cuda.synchronize(dev)
+
+    def _config(self):
+        return (self.n_blocks, self.B, self.H, self.d, self.n["text"], self.n["ref"], self.n["tgt"],
+                self.log_steps, self.mpl, self.cue, self.sample_stride, self.mass_rows, self.diagnostics)
+
+    def trace(self, n_steps):
+        """The observation record of the logged steps 0 .. n_steps - 1 (read
+        after they have run): per (step, block) the mode and gbar of every
+        sample, the head-mean exposure the gate read (Eq. 5 on M_{t-1}; None at
+        t = 0) and a_b now. A list of dicts, one per (step, block), for a JSONL
+        log; one host read of the logs."""
+        T = int(n_steps)
+        if T < 1 or T > self.log_steps:
+            raise ValueError("trace: need 1 <= n_steps <= log_steps (%d)" % self.log_steps)
+        modes = self.modes[:T].cpu().tolist()
+        gbar = self.gbar[:T].double().cpu().tolist()
+        mbar = self.M[:T].double().mean(-1).cpu().tolist()
+        a_b = self.a_b.cpu().tolist()
+        out = []
+        for t in range(T):
+            for b in range(self.n_blocks):
+                out.append({"t": t, "b": b, "mode": modes[t][b],
+                            "gbar": [None if g != g else g for g in gbar[t][b]],
+                            "m_bar_read": mbar[t][b] if t >= 1 else None, "a_b": a_b[b]})
+        return out
 
     def check(self, stream=None):
         api.refadapt_check_error(self.err, stream)

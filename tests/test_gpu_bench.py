@@ -16,8 +16,9 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def test_bench_line_on_the_single_block_workload(cuda_ok, tmp_path):
     out = tmp_path / "line.json"
+    trace = tmp_path / "trace.jsonl"
     cmd = [sys.executable, os.path.join(ROOT, "bench.py"), "--config", "c1", "--steps", "4", "--warmup", "3",
-           "--no-dit", "--cpu-budget-s", "2", "--out", str(out)]
+           "--no-dit", "--cpu-budget-s", "2", "--out", str(out), "--trace", str(trace), "--nvtx"]
     res = subprocess.run(cmd, cwd=ROOT, capture_output=True, text=True, timeout=600)
     assert res.returncode == 0, res.stderr[-2000:]
     lines = [ln for ln in res.stdout.splitlines() if ln.startswith("{")]
@@ -36,6 +37,14 @@ def test_bench_line_on_the_single_block_workload(cuda_ok, tmp_path):
     e2e = line["e2e"]
     assert e2e["value"] > 0 and e2e["h2d_bytes_per_step"] > 0 and e2e["d2h_bytes_per_step"] > 0, e2e
     assert line["e2e_unpadded"]["value"] > 0
+    # the observation record of the trajectory: one line per (step, block)
+    recs = [json.loads(x) for x in trace.read_text().splitlines()]
+    cfg = line["config"]
+    assert len(recs) == cfg["trajectory_steps"] * cfg["blocks"]
+    assert {tuple(sorted(r)) for r in recs} == {("a_b", "b", "gbar", "m_bar_read", "mode", "t")}
+    by_t = {r["t"]: r["mode"][0] for r in recs if r["b"] == 0}
+    assert [by_t[int(t)] for t in sorted(line["modes_per_step"], key=int)] == \
+        [line["modes_per_step"][t][0] for t in sorted(line["modes_per_step"], key=int)]
 
 
 def test_bench_separate_cache_update_schedule(cuda_ok):
