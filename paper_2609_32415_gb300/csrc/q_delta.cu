@@ -327,7 +327,8 @@ struct ClusterParams {
   float eps;
   float* d_out;
   uint64_t budget_ns;
-  // refadapt_q_delta_gate: the last cluster to write its D runs the gate
+  // refadapt_q_delta_gate: each leader stores its head's score term and takes
+  // a ticket; the leader that takes the last one decides for the block
   int32_t fuse_gate;
   uint32_t* gate_ticket;  // workspace counter (zero between launches)
   float2* gate_terms;     // workspace [B * H]: each head's score term (g, e)
