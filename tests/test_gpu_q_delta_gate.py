@@ -68,10 +68,14 @@ CASES = [
     (3, 4, 515, 64, 5),
     # slabs too long for one cluster: the multi-block path, the gate as a second launch
     (1, 2, 100000, 128, 4),
+    # one row, one head
+    (1, 1, 1, 64, 1),
+    # more slabs than clusters fit at once: the multi-block path
+    (4, 40, 300, 128, 3),
 ]
 
 
-@pytest.mark.parametrize("B,H,n,d,L", CASES, ids=["24heads", "B2", "d64", "multiblock"])
+@pytest.mark.parametrize("B,H,n,d,L", CASES, ids=["24heads", "B2", "d64", "multiblock", "one-row", "160slabs"])
 @pytest.mark.parametrize("cue", [0, 1, 2], ids=["product", "change", "exposure"])
 def test_fused_gate_equals_two_calls(cuda_ok, B, H, n, d, L, cue):
     T, nb = 3, 3
