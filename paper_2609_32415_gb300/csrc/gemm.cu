@@ -63,12 +63,16 @@ constexpr int TMEM_COLS = 512;
 static_assert(SMEM_ALLOC <= 232448, "shared memory budget");
 
 // CTA-pair kernel: 256 x 256 output tiles; each CTA stages its 128 rows of A
-// and its 128-column half of the W tile (32 KB per stage, 6 stages; a
-// seventh stage measured no faster).
+// and its 128-column half of the W tile, 128 of K per stage (two 128-byte
+// swizzle chunks per operand, 64 KB per stage, 3 stages): half the stage
+// hand-offs of 64-wide stages, which the fused epilogues gained from (GELU
+// +3 %); a K % 128 == 64 tail is a half stage.
 constexpr int P_TM = 256;
-constexpr int P_STAGES = 6;
-constexpr int P_A_BYTES = 128 * BK * 2;
-constexpr int P_B_BYTES = 128 * BK * 2;
+constexpr int P_STAGES = 3;
+constexpr int P_BK = 128;              // K per stage: two 64-column chunks per operand
+constexpr int P_CHUNK = 128 * 64 * 2;  // 128 rows x 64 K of one operand (one 128-byte swizzle span)
+constexpr int P_A_BYTES = 128 * P_BK * 2;
+constexpr int P_B_BYTES = 128 * P_BK * 2;
 constexpr int P_STAGE_BYTES = P_A_BYTES + P_B_BYTES;
 constexpr int P_OFF_BAR = P_STAGES * P_STAGE_BYTES;
 constexpr int P_NUM_BARS = 2 * P_STAGES + 2 + 2 + 1;
@@ -462,13 +466,18 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_pair_kernel(const __grid_cons
       for (int64_t t = cid; ok && t < p.total_tiles; t += ncl) {
         const Tile tl = decode<P_TM>(p, t);
         if (!tl.live) continue;
-        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+        for (int kb = 0; kb < (p.kblocks + 1) / 2; ++kb, ++it) {
           const int st = int(it % P_STAGES);
           if (it >= P_STAGES && !(ok = mbar_wait(empty + st, uint32_t((it / P_STAGES - 1) & 1), ctl))) break;
           uint8_t* sa = smem + st * P_STAGE_BYTES;
-          if (rank == 0) mbar_arrive_expect_tx(full + st, 2 * P_STAGE_BYTES);
-          tma_load_4d_pair(sa, &p.tm_a[tl.seg], full0 + 8u * st, kb * BK, tl.m0 + int(rank) * 128, 0, tl.s);
-          tma_load_4d_pair(sa + P_A_BYTES, &p.tm_w[tl.seg], full0 + 8u * st, kb * BK, tl.n0 + int(rank) * 128, 0, 0);
+          const int chunks = (2 * kb + 1 < p.kblocks) ? 2 : 1;  // K % 128 == 64: the last stage is half
+          if (rank == 0) mbar_arrive_expect_tx(full + st, 4 * chunks * P_CHUNK);
+          for (int c = 0; c < chunks; ++c) {
+            tma_load_4d_pair(sa + c * P_CHUNK, &p.tm_a[tl.seg], full0 + 8u * st, kb * P_BK + c * 64,
+                             tl.m0 + int(rank) * 128, 0, tl.s);
+            tma_load_4d_pair(sa + P_A_BYTES + c * P_CHUNK, &p.tm_w[tl.seg], full0 + 8u * st, kb * P_BK + c * 64,
+                             tl.n0 + int(rank) * 128, 0, 0);
+          }
         }
       }
       if (*abort_flag) {
@@ -501,15 +510,19 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_pair_kernel(const __grid_cons
         if (use > 0 && !(ok = mbar_wait_cluster(tempty + buf, uint32_t((use - 1) & 1), ctl))) break;
         tc_fence_after();
         const uint32_t d_t = tmem + uint32_t(buf * BN);
-        for (int kb = 0; kb < p.kblocks; ++kb, ++it) {
+        for (int kb = 0; kb < (p.kblocks + 1) / 2; ++kb, ++it) {
           const int st = int(it % P_STAGES);
           if (!(ok = mbar_wait(full + st, uint32_t((it / P_STAGES) & 1), ctl))) break;
           tc_fence_after();
           const uint32_t sa = s0 + st * P_STAGE_BYTES, sb = sa + P_A_BYTES;
+          const int ksteps = (2 * kb + 1 < p.kblocks) ? P_BK / 16 : 64 / 16;
 #pragma unroll
-          for (int kk = 0; kk < BK / 16; ++kk)
-            umma_ss_pair(d_t, sdesc_sw128(sa + kk * 32, 16, 1024), sdesc_sw128(sb + kk * 32, 16, 1024), IDESC,
+          for (int kk = 0; kk < P_BK / 16; ++kk) {
+            if (kk >= ksteps) break;
+            const uint32_t o = uint32_t((kk >> 2) * P_CHUNK + (kk & 3) * 32);
+            umma_ss_pair(d_t, sdesc_sw128(sa + o, 16, 1024), sdesc_sw128(sb + o, 16, 1024), IDESC,
                          (kb > 0 || kk > 0) ? 1u : 0u);
+          }
           umma_commit_pair(empty + st, 0x3);
           issued = true;
         }

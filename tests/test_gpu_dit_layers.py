@@ -122,7 +122,7 @@ TILE_MODES = [1, 2]
 
 @pytest.mark.parametrize("tile_mode", TILE_MODES)
 @pytest.mark.parametrize("K,N,rows", [(64, 256, [1]), (256, 768, [40, 130, 77]), (3072, 512, [300]),
-                                      (512, 2048, [2500]), (128, 512, [4500, 70])])
+                                      (512, 2048, [2500]), (128, 512, [4500, 70]), (192, 512, [700])])
 def test_gemm_store_matches_oracle(cuda_ok, K, N, rows, tile_mode):
     """Tiles are numbered in bands of 16 tile rows: 4500 rows make a full band
     and a partial one of 256-row tiles (18 = 16 + 2) and of 128-row tiles
